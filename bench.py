@@ -1,0 +1,325 @@
+"""Benchmark of batched TFHE programmable bootstrapping on GB300.
+
+One step = one rosetta_pbs_batch call over the whole batch (modulus switch,
+blind rotation, sample extraction, key switch) with keys and inputs resident
+in HBM.  Default workload: the standard parameter set (n=742, k=1, N=2048,
+PBS base 2^23 x 1, KS base 2^3 x 5) on a batch of 4096 ciphertexts with a
+4-bit GELU LUT.
+
+Prints one JSON line (rank 0).  `--impl reference` times the CPU oracle on
+the host cores instead (the reference arm: a deliberately plain program).
+"""
+
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import workload as W  # noqa: E402
+
+METRIC = "PBS/sec (blind rotate + key switch) on 1 GB300; fraction of roofline"
+UNIT = "PBS/s"
+
+
+def describe(p, batch):
+    return (f"{p.name}: n={p.n} k={p.k} N={p.N} PBS base 2^{p.pbs_base_log} x {p.pbs_level}, "
+            f"KS base 2^{p.ks_base_log} x {p.ks_level}, {p.msg_bits}-bit LUT {p.lut[0]}, batch {batch}")
+
+
+# ---------------------------------------------------------------------------- op counts
+
+def min_primes(p) -> int:
+    """Smallest number of 31-bit primes whose product exceeds twice the
+    largest integer value of an external-product coefficient."""
+    bits = 63 + (p.pbs_base_log - 1) + math.log2((p.k + 1) * p.pbs_level * p.N) + 1
+    return math.ceil(bits / 31)
+
+
+def int_ops_per_pbs(p):
+    """Algorithmic 32-bit integer operations of one PBS: (blind rotation,
+    key switch).  Counting convention: NTT butterflies 8 ops, pointwise
+    multiply-accumulate 6, CRT 10 per prime, decomposition 6 per level,
+    rotation/accumulate 4, per coefficient; key switch 3 per digit x word."""
+    P = min_primes(p)
+    k1, l, N = p.k + 1, p.pbs_level, p.N
+    per_cmux = ((k1 * l + k1) * P * (N // 2) * int(math.log2(N)) * 8 + k1 * l * k1 * P * N * 6
+                + k1 * N * 10 * P + k1 * N * l * 6 + k1 * N * 4)
+    ks = p.kN * p.ks_level * (p.n + 1) * 3 + p.kN * p.ks_level * 6
+    return per_cmux * p.n, ks
+
+
+def peaks():
+    try:
+        return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except OSError:
+        return {}
+
+
+# ---------------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *a):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 8:
+                continue
+            try:
+                sm.append(float(f[0]))
+                mx = float(f[1])
+            except ValueError:
+                continue
+            for name, v in zip(names, f[4:8]):
+                if v.lower() == "active":
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------- oracle (CPU) timing
+
+def oracle_pbs_rate(p, count, threads=None, seed=0):
+    """PBS/s of the CPU oracle on `count` ciphertexts with uniform-word keys."""
+    import oracle as O
+    bsk, ksk = W.uniform_keys(p)
+    lwe = W.uniform_ciphertexts(p, count, sub=1000 + seed)
+    lut = W.lut_torus(p)
+    t = threads or O.default_threads()
+    t0 = time.perf_counter()
+    O.pbs_batch(p, bsk, ksk, lwe, lut, threads=t)
+    dt = time.perf_counter() - t0
+    return count / dt, dt, t
+
+
+def run_reference(args, p, batch):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    import oracle as O
+    O.build()
+    cores = O.default_threads()
+    sample = max(1, min(batch, cores))
+    for _ in range(args.warmup):
+        oracle_pbs_rate(p, 1, threads=1)
+    rates, times = [], []
+    for s in range(args.steps):
+        r, dt, t = oracle_pbs_rate(p, sample, threads=cores, seed=s)
+        rates.append(r)
+        times.append(dt)
+    value = sample * len(times) / sum(times)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * sum(times) / len(times),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u64", "data": "synthetic",
+        "config": {"workload": describe(p, batch), "batch": batch, "keys": "uniform words"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": f"{sample} ciphertexts of the workload per step (schoolbook CPU oracle)"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------------------- GPU arm
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", default="standard", choices=sorted(W.CONFIGS))
+    ap.add_argument("--batch", type=int, default=0, help="override the workload's batch")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-sample", type=int, default=0, help="oracle sample size (default: host cores)")
+    args = ap.parse_args()
+    p = W.CONFIGS[args.config]
+    batch = args.batch or p.batch
+    if args.impl == "reference":
+        return run_reference(args, p, batch)
+
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", init_method="env://")
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+
+    import paper_2609_16915_gb300 as R
+    R.load()
+
+    def d(a):
+        return torch.from_numpy(np.ascontiguousarray(a).view(np.int64)).to(dev)
+
+    # workload: uniform-word keys (indistinguishable from real keys; the cost
+    # does not depend on key values) and uniform ciphertexts, all resident
+    bsk, ksk = W.uniform_keys(p)
+    lwe = d(W.uniform_ciphertexts(p, batch, sub=rank))
+    lut = d(W.lut_torus(p))
+    out = torch.empty((batch, p.n + 1), dtype=torch.int64, device=dev)
+    big = torch.empty((batch, p.kN + 1), dtype=torch.int64, device=dev)
+    ctx = R.Context(p, device=local, max_batch=batch)
+    ctx.upload_bsk(d(bsk))
+    ctx.upload_ksk(d(ksk))
+    del bsk, ksk
+    stream = torch.cuda.current_stream(dev)
+    ctx.sync_status(stream)
+    flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.int32, device=dev)  # 256 MB > L2
+
+    def barrier():
+        if dist:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    for _ in range(max(3, args.warmup)):
+        ctx.pbs_batch(lwe, lut, out, stream)
+    ctx.sync_status(stream)
+
+    # timed region: K steps, each bracketed by events; L2 flushed between steps
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    barrier()
+    with ClockSampler(local) as clk:
+        wall0 = time.perf_counter()
+        for s in range(args.steps):
+            flush.zero_()
+            ev[s][0].record(stream)
+            ctx.pbs_batch(lwe, lut, out, stream)
+            ev[s][1].record(stream)
+        barrier()
+        wall = time.perf_counter() - wall0
+    ctx.sync_status(stream)
+    step_ms = [a.elapsed_time(b) for a, b in ev]
+    total_ms = sum(step_ms)
+    t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
+    if dist:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    total_ms = float(t.item())
+    value = world * batch * args.steps / (total_ms / 1e3)
+
+    # dominant kernel (blind rotation) alone, same launch, events on its stream
+    br_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(3)]
+    ks_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(3)]
+    for i in range(3):
+        flush.zero_()
+        br_ev[i][0].record(stream)
+        ctx.blind_rotate_extract_batch(lwe, lut, big, stream)
+        br_ev[i][1].record(stream)
+        flush.zero_()
+        ks_ev[i][0].record(stream)
+        ctx.keyswitch_batch(big, out, stream)
+        ks_ev[i][1].record(stream)
+    ctx.sync_status(stream)
+    br_ms = statistics.mean(a.elapsed_time(b) for a, b in br_ev)
+    ks_ms = statistics.mean(a.elapsed_time(b) for a, b in ks_ev)
+
+    # end to end through the public API with pinned host buffers
+    h_in = torch.from_numpy(W.uniform_ciphertexts(p, batch, sub=rank).view(np.int64)).pin_memory()
+    h_out = torch.empty((batch, p.n + 1), dtype=torch.int64).pin_memory()
+    h_lut = torch.from_numpy(W.lut_torus(p).view(np.int64)).pin_memory()
+    ctx.pbs_batch(h_in, h_lut, h_out, stream)
+    barrier()
+    e2e_steps = max(1, min(args.steps, 5))
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        ctx.pbs_batch(h_in, h_lut, h_out, stream)   # copies in, PBS, copies out, synchronises
+    e2e_s = (time.perf_counter() - t0) / e2e_steps
+    e2e_t = torch.tensor([e2e_s], dtype=torch.float64, device=dev)
+    if dist:
+        dist.all_reduce(e2e_t, op=dist.ReduceOp.MAX)
+    e2e_value = world * batch / float(e2e_t.item())
+
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    pk = peaks()
+    sm_max = pk.get("sm_max_mhz", 2070.0)
+    alu_peak = sms * 128 * sm_max * 1e6 / 1e12   # T int32 ops/s: SMs x 128 lanes x max clock
+    br_ops, ks_ops = int_ops_per_pbs(p)
+    achieved = br_ops * batch / (br_ms / 1e3) / 1e12
+    pbs_roof = alu_peak * 1e12 / (br_ops + ks_ops)
+
+    if rank != 0:
+        if dist:
+            dist.destroy_process_group()
+        return
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": max(3, args.warmup), "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "u64", "data": "synthetic",
+        "config": {"workload": describe(p, batch), "batch": batch, "parallelism": f"dp{world}" if world > 1 else "none",
+                   "l2": "flushed between steps (256 MB write)", "keys": "uniform words, resident"},
+        "roofline": {"bound": "alu", "kernel": "blind_rotate_kernel", "achieved": achieved, "peak": alu_peak,
+                     "unit": "Tops/s (int32)", "frac": achieved / alu_peak, "traffic": None,
+                     "peak_basis": f"{sms} SMs x 128 int32 lanes x {sm_max:.0f} MHz (sm_max_mhz of MEASURED_PEAKS.json)",
+                     "kernel_ms": br_ms, "keyswitch_ms": ks_ms,
+                     "pbs_roof": pbs_roof, "pbs_frac_of_roof": value / world / pbs_roof},
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": batch * (p.n + 1) * 8 + lut.numel() * 8,
+                "d2h_bytes_per_step": batch * (p.n + 1) * 8},
+        "gpu_launches": 2 * args.steps,
+        "clocks": clk.summary(),
+        "wall_s_timed": wall,
+    }
+    if not args.no_cpu_baseline:
+        import oracle as O
+        O.build()
+        cores = O.default_threads()
+        sample = args.cpu_sample or cores
+        r, dt, t = oracle_pbs_rate(p, sample, threads=cores)
+        line["cpu_baseline"] = {"value": r, "unit": UNIT, "cores": t, "kind": "oracle",
+                                "sample": f"{sample} ciphertexts of the workload, uniform-word keys, {dt:.1f} s"}
+    print(json.dumps(line), flush=True)
+    if dist:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,145 @@
+/*
+ * rosetta.h — C ABI of the GB300 (sm_103a) batched TFHE programmable
+ * bootstrapping library (librosetta.so).
+ *
+ * What it computes.  The paper (Background, "TFHE Scheme") states the
+ * primitive as
+ *     [[f(m)]] = TFHE-LUT_f([[m]])
+ * for an LWE ciphertext [[m]] in Z_q^{n+1} and a look-up table f whose
+ * entries are written into the coefficients of a test polynomial; blind
+ * rotation by the encrypted index followed by extraction of the constant
+ * term yields a fresh LWE encryption of f(m).  This library evaluates that
+ * primitive for a whole batch of independent ciphertexts, with q = 2^64:
+ *   1. modulus switch of every word to Z_{2N} (round half up);
+ *   2. blind rotation of the test polynomial through n CMux steps, each a
+ *      GGSW x GLWE external product (signed gadget decomposition, then exact
+ *      negacyclic products in Z_{2^64}[X]/(X^N+1));
+ *   3. sample extraction of the constant coefficient (LWE of dimension kN);
+ *   4. LWE key switch back to dimension n.
+ * Outputs are bit-identical to the plain definition (schoolbook products mod
+ * 2^64), not approximations.
+ *
+ * Word layout.  All ciphertext and key words are uint64 torus elements.
+ *   LWE ciphertext   [a_0 .. a_{n-1}, b], phase = b - <a, s>
+ *   batch of LWEs    row-major [batch][n+1]
+ *   raw BSK          [n][(k+1)*l][k+1][N]; BSK_i is the GGSW of the LWE key
+ *                    bit s_i: row r = j*l + (lev-1) is a GLWE encryption of
+ *                    0 with s_i * 2^(64 - lev*beta) added to the constant
+ *                    coefficient of component j (j = k is the body)
+ *   raw KSK          [kN][l_ks][n+1]; row [i][lev] is an LWE encryption under
+ *                    the output key of s'_i * 2^(64 - lev*beta_ks), s' the
+ *                    extracted GLWE key (s'_{jN+t} = S_j[t])
+ *   LUT              2^p torus words lut[m] = Delta * f(m), Delta = 2^(63-p)
+ *                    (one padding bit); the test polynomial is
+ *                    v[t] = lut[(t + h)/box] for t < N - h and -lut[0] above,
+ *                    box = N / 2^p, h = box / 2
+ *
+ * Pointers and ownership.  The caller owns every buffer it passes and the
+ * stream.  Ciphertext and LUT pointers may be device memory or host memory
+ * (pinned or pageable); host buffers are staged through library-owned device
+ * buffers with copies on the same stream.  Buffers must be 8-byte aligned.
+ * Input and output ranges must not overlap.  The library owns the transformed
+ * keys, twiddle tables and scratch; rosetta_destroy frees them.
+ *
+ * Streams and errors.  `stream` is a cudaStream_t passed as void* (NULL =
+ * the legacy default stream).  Calls that launch work are asynchronous with
+ * respect to the host when every buffer is device memory; with host buffers
+ * they return after the copy back has completed.  Every function returns a
+ * rosetta_status; argument errors are detected before anything is enqueued.
+ * Execution errors surface at rosetta_sync_status or at the next call.
+ * No function falls back to the CPU.
+ *
+ * Threading.  A context may be used from one host thread at a time.
+ */
+#ifndef ROSETTA_H
+#define ROSETTA_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  ROSETTA_OK = 0,
+  ROSETTA_ERR_INVALID_ARG = -1,        /* NULL, misaligned, aliasing, bad size, batch too large */
+  ROSETTA_ERR_UNSUPPORTED_PARAMS = -2, /* parameter set the kernels do not cover */
+  ROSETTA_ERR_KEYS_MISSING = -3,       /* BSK or KSK not uploaded */
+  ROSETTA_ERR_CUDA = -4,               /* a CUDA runtime call or launch failed */
+  ROSETTA_ERR_OOM = -5,                /* device allocation failed */
+  ROSETTA_ERR_TIMEOUT = -6             /* a bounded device-side wait expired */
+} rosetta_status;
+
+typedef struct rosetta_ctx rosetta_ctx; /* opaque, library-owned */
+
+typedef struct {
+  uint32_t lwe_dim;      /* n: dimension of input and output LWE ciphertexts */
+  uint32_t glwe_dim;     /* k: GLWE dimension (the kernels support k = 1) */
+  uint32_t poly_size;    /* N: power of two, 256 .. 8192 */
+  uint32_t pbs_base_log; /* beta: PBS gadget base 2^beta, 1 .. 28 */
+  uint32_t pbs_level;    /* l: PBS gadget levels, beta*l <= 64 */
+  uint32_t ks_base_log;  /* beta_ks: key-switch gadget base, 1 .. 16 */
+  uint32_t ks_level;     /* l_ks: key-switch levels, beta_ks*l_ks <= 64 */
+  uint32_t msg_bits;     /* p: LUT entries 2^p; N / 2^p must be >= 2 */
+  uint32_t max_batch;    /* staging/scratch capacity in ciphertexts; 0 = grow on demand */
+} rosetta_params;
+
+/* Create a context on CUDA device `cuda_device` for parameter set *p.
+ * Computes the NTT primes' twiddle tables and CRT constants and allocates
+ * scratch for p->max_batch ciphertexts.  *out receives the context (NULL on
+ * error).  Errors: INVALID_ARG (NULL), UNSUPPORTED_PARAMS, CUDA, OOM. */
+int rosetta_params_init(rosetta_ctx **out, const rosetta_params *p, int cuda_device);
+
+/* Upload the raw bootstrapping key (layout above, n_words =
+ * n*(k+1)*l*(k+1)*N) and convert it on the device to the transform domain
+ * used by the external product (per-prime negacyclic NTT of the centred
+ * words).  The source may be host or device memory (src_is_device selects);
+ * the caller keeps ownership and may free it after the call returns.  The
+ * conversion is stream-ordered on `stream`.  Errors: INVALID_ARG, CUDA, OOM. */
+int rosetta_upload_bsk(rosetta_ctx *ctx, const uint64_t *bsk, size_t n_words,
+                       int src_is_device, void *stream);
+
+/* Upload the raw key-switching key (n_words = kN*l_ks*(n+1)); same source
+ * rules as rosetta_upload_bsk.  Errors: INVALID_ARG, CUDA, OOM. */
+int rosetta_upload_ksk(rosetta_ctx *ctx, const uint64_t *ksk, size_t n_words,
+                       int src_is_device, void *stream);
+
+/* Programmable bootstrapping of `batch` ciphertexts:
+ *   lwe_in  [batch][n+1]  input ciphertexts
+ *   lut     [2^p]         torus LUT words (Delta * f(m))
+ *   lwe_out [batch][n+1]  PBS outputs (modulus switch, blind rotation,
+ *                         sample extraction, key switch)
+ * batch == 0 is a no-op returning OK.  Errors: INVALID_ARG, KEYS_MISSING,
+ * CUDA, OOM. */
+int rosetta_pbs_batch(rosetta_ctx *ctx, const uint64_t *lwe_in, uint32_t batch,
+                      const uint64_t *lut, uint64_t *lwe_out, void *stream);
+
+/* The first three steps of rosetta_pbs_batch only: writes the extracted
+ * ciphertexts of dimension kN, lwe_big_out [batch][kN+1].  Needs the BSK. */
+int rosetta_blind_rotate_extract_batch(rosetta_ctx *ctx, const uint64_t *lwe_in, uint32_t batch,
+                                       const uint64_t *lut, uint64_t *lwe_big_out, void *stream);
+
+/* LWE key switch of `batch` ciphertexts of dimension kN, lwe_big_in
+ * [batch][kN+1], to dimension n, lwe_out [batch][n+1]:
+ *   out = (0, .., 0, b') - sum_i sum_lev d_{i,lev}(a'_i) * KSK[i][lev]
+ * with d the signed base-2^beta_ks digits of a'_i rounded to its top
+ * beta_ks*l_ks bits.  Needs the KSK. */
+int rosetta_keyswitch_batch(rosetta_ctx *ctx, const uint64_t *lwe_big_in, uint32_t batch,
+                            uint64_t *lwe_out, void *stream);
+
+/* Wait for all work on `stream` and report any deferred execution error
+ * (CUDA, TIMEOUT).  Returns OK when the stream finished cleanly. */
+int rosetta_sync_status(rosetta_ctx *ctx, void *stream);
+
+/* Free everything the context owns.  Waits for the context's device work.
+ * NULL is ignored. */
+void rosetta_destroy(rosetta_ctx *ctx);
+
+/* Static string naming a status code. */
+const char *rosetta_status_string(int status);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* ROSETTA_H */

@@ -1,0 +1,268 @@
+// Blind rotation (modulus switch -> n CMux steps -> sample extraction) for a
+// batch of LWE ciphertexts, one thread-block cluster of four CTAs per
+// ciphertext.
+//
+// Construction (Background, "TFHE Scheme", PBS): the LUT is written into a
+// test polynomial v, the accumulator starts as the trivial GLWE
+// (0, X^{-b~} v) and every CMux step i multiplies it by X^{a~_i s_i} through
+// the external product with the GGSW BSK_i:
+//     ACC <- ACC + BSK_i (x) (X^{a~_i} ACC - ACC).
+// The external product decomposes each coefficient of the rotated difference
+// into signed digits and forms sum_r D_r * BSK_i[r][c] in Z_{2^64}[X]/(X^N+1).
+// Those products are computed exactly: the integer value of every output
+// coefficient is below M/2 with M the product of four 29-bit NTT primes, so
+// four negacyclic NTTs, a pointwise multiply-accumulate per prime and an
+// explicit CRT (X = sum_q y_q M/p_q - round(sum_q y_q/p_q) M, evaluated mod
+// 2^64) give the same words as the schoolbook product.
+//
+// Work split.  CTA r of the cluster (r = 0..3) does all transforms for prime
+// r and owns coefficients [rN/4, (r+1)N/4) of both accumulator polynomials.
+// One CMux step is three phases separated by cluster barriers:
+//   1. each owner forms the rotated difference for its quarter (reading the
+//      rotated source coefficient from whichever CTA owns it, through
+//      distributed shared memory) and writes its gadget digits locally;
+//   2. each prime-CTA gathers all digits, runs forward NTTs two polynomials at
+//      a time, multiplies by the transform-domain BSK_i (streamed from
+//      global memory with 16-byte loads, Montgomery form), runs the two
+//      inverse NTTs and sends each owner the CRT-scaled residues of its
+//      quarter;
+//   3. each owner combines the four residues of its coefficients (explicit
+//      CRT) and adds the result to the accumulator.
+#include <cooperative_groups.h>
+
+#include <type_traits>
+
+#include "internal.h"
+#include "ntt.cuh"
+
+namespace rosetta {
+namespace cg = cooperative_groups;
+
+template <int LOGN>
+struct BrShape {
+  static constexpr int N = 1 << LOGN;
+  static constexpr int T = N / 8;
+  static constexpr int Q = N / 4;                      // coefficients owned per CTA
+  static constexpr int XBUF = (LOGN <= 11) ? 2 : 1;    // exchange buffers (polys)
+};
+
+template <int LOGN, bool DIG16>
+__global__ void __launch_bounds__((1 << LOGN) / 8) blind_rotate_kernel(const BrArgs a) {
+  using S = NttShape<LOGN>;
+  using B = BrShape<LOGN>;
+  using DigT = typename std::conditional<DIG16, int16_t, int32_t>::type;
+  constexpr uint32_t N = B::N, T = B::T, Q = B::Q;
+  constexpr uint32_t TWO_N = 2 * N;
+
+  cg::cluster_group cluster = cg::this_cluster();
+  const uint32_t rank = cluster.block_rank();
+  const uint32_t ct = blockIdx.x / 4;
+  const uint32_t tau = threadIdx.x;
+
+  extern __shared__ __align__(16) unsigned char smem[];
+  uint2 *tw = reinterpret_cast<uint2 *>(smem);                   // [N]
+  uint64_t *acc = reinterpret_cast<uint64_t *>(tw + N);          // [2][Q]
+  uint32_t *res = reinterpret_cast<uint32_t *>(acc + 2 * Q);     // [4 primes][2][Q]
+  uint32_t *xb = res + kPrimes * 2 * Q;                          // [XBUF][XB_WORDS]
+  DigT *dig = reinterpret_cast<DigT *>(xb + B::XBUF * S::XB_WORDS);  // [2l][Q]
+  uint16_t *atil = reinterpret_cast<uint16_t *>(dig + 2 * a.level * Q);  // [n+1]
+
+  const uint32_t p = a.cc.pr[rank].p;
+  const uint32_t p_inv = a.cc.pr[rank].p_inv;
+  const uint32_t crt_c = a.cc.pr[rank].crt_c;
+  const uint32_t crt_cs = a.cc.pr[rank].crt_cs;
+
+  // ---- set-up: twiddles, modulus switch, accumulator ----
+  for (uint32_t m = tau; m < N; m += T) tw[m] = a.tw[rank * N + m];
+  const uint64_t *lwe = a.lwe_in + static_cast<size_t>(ct) * (a.n + 1);
+  constexpr uint32_t SH = 63 - LOGN;  // 64 - log2(2N)
+  for (uint32_t i = tau; i <= a.n; i += T)
+    atil[i] = static_cast<uint16_t>(((lwe[i] + (1ull << (SH - 1))) >> SH) & (TWO_N - 1));
+  __syncthreads();
+  {
+    const uint32_t btil = atil[a.n];
+    const uint32_t box = N >> a.msg_bits, h = box >> 1;
+#pragma unroll
+    for (int m = 0; m < 4; ++m) {
+      const uint32_t item = tau + m * T;
+      const uint32_t c = item / Q, jl = item % Q, j = rank * Q + jl;
+      if (c == 0) {
+        acc[jl] = 0;
+      } else {
+        // (X^{2N - b~} v)[j] = +-v[t], t = (j + b~) mod 2N folded into [0, N)
+        const uint32_t e = (j + btil) & (TWO_N - 1);
+        const uint32_t t = e & (N - 1);
+        const uint64_t v = (t < N - h) ? a.lut[(t + h) / box] : (0ull - a.lut[0]);
+        acc[Q + jl] = (e >= N) ? 0ull - v : v;
+      }
+    }
+  }
+  cluster.sync();
+
+  const uint64_t *racc[kPrimes];
+  const DigT *rdig[kPrimes];
+  uint32_t *rres[kPrimes];
+#pragma unroll
+  for (int o = 0; o < kPrimes; ++o) {
+    racc[o] = cluster.map_shared_rank(acc, o);
+    rdig[o] = cluster.map_shared_rank(dig, o);
+    rres[o] = cluster.map_shared_rank(res, o);
+  }
+  const uint32_t L2 = 2 * a.level;
+  const uint32_t bits = a.base_log * a.level;
+  const uint64_t Bmask = (1ull << a.base_log) - 1;
+  const uint64_t Bhalf = 1ull << (a.base_log - 1);
+  const uint64_t round_add = bits >= 64 ? 0 : (1ull << (63 - bits));
+  const uint32_t round_sh = bits >= 64 ? 0 : 64 - bits;
+
+  for (uint32_t i = 0; i < a.n; ++i) {
+    const uint32_t at = atil[i];
+    if (at == 0) continue;  // X^0 ACC - ACC = 0: the step adds nothing
+
+    // ---- phase 1: rotated difference and gadget digits of the owned quarter ----
+#pragma unroll
+    for (int m = 0; m < 4; ++m) {
+      const uint32_t item = tau + m * T;
+      const uint32_t c = item / Q, jl = item % Q, j = rank * Q + jl;
+      uint32_t e = (j + TWO_N - at) & (TWO_N - 1);  // (X^a P)[j] = +-P[(j - a) mod 2N]
+      const bool neg = e >= N;
+      e &= N - 1;
+      uint64_t v = racc[e / Q][c * Q + (e % Q)];
+      if (neg) v = 0ull - v;
+      const uint64_t diff = v - acc[c * Q + jl];
+      uint64_t cv = bits >= 64 ? diff : (diff + round_add) >> round_sh;
+      for (int l = static_cast<int>(a.level) - 1; l >= 0; --l) {
+        const uint64_t d = cv & Bmask;
+        cv >>= a.base_log;
+        int32_t ds = static_cast<int32_t>(d);
+        if (d >= Bhalf) {
+          ds -= static_cast<int32_t>(Bmask + 1);
+          cv += 1;
+        }
+        dig[(c * a.level + l) * Q + jl] = static_cast<DigT>(ds);
+      }
+    }
+    cluster.sync();
+
+    // ---- phase 2: transforms and pointwise products for prime `rank` ----
+    uint32_t oh[2][8];
+    const uint32_t *gbase = a.bsk + (static_cast<size_t>(i) * kPrimes + rank) * (static_cast<size_t>(L2) * 2 * N);
+    for (uint32_t r0 = 0; r0 < L2; r0 += 2) {
+      uint32_t x[2][8];
+#pragma unroll
+      for (int pp = 0; pp < 2; ++pp)
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          const int32_t d = rdig[q >> 1][(r0 + pp) * Q + tau + (q & 1) * T];
+          x[pp][q] = static_cast<uint32_t>(d + static_cast<int32_t>(p));  // in (0, 2p)
+        }
+      ntt_forward<LOGN, 2, B::XBUF>(x, tw, xb, tau, p);
+#pragma unroll
+      for (int c = 0; c < 2; ++c) {
+        const uint4 *g0 = reinterpret_cast<const uint4 *>(gbase + (static_cast<size_t>(r0) * 2 + c) * N + 8 * tau);
+        const uint4 *g1 = reinterpret_cast<const uint4 *>(gbase + (static_cast<size_t>(r0 + 1) * 2 + c) * N + 8 * tau);
+        const uint4 a0 = __ldg(g0), a1 = __ldg(g0 + 1), b0 = __ldg(g1), b1 = __ldg(g1 + 1);
+        const uint32_t ga[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+        const uint32_t gb[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          // forward outputs < 8p, brought below 4p; BSK words < p in Montgomery
+          // form, so the pair sum stays below p * 2^32
+          const uint32_t x0 = cond_sub(x[0][e], 4 * p), x1 = cond_sub(x[1][e], 4 * p);
+          const uint64_t prod = static_cast<uint64_t>(x0) * ga[e] + static_cast<uint64_t>(x1) * gb[e];
+          const uint32_t rr = redc(prod, p, p_inv);  // (0, 2p)
+          oh[c][e] = (r0 == 0) ? rr : cond_sub(oh[c][e] + rr, 4 * p);
+        }
+      }
+    }
+    ntt_inverse<LOGN, 2, B::XBUF>(oh, tw, xb, tau, p);
+#pragma unroll
+    for (int c = 0; c < 2; ++c)
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const uint32_t y = shoup_mul(oh[c][q], crt_c, crt_cs, p);  // [0, 2p)
+        rres[q >> 1][(rank * 2 + c) * Q + tau + (q & 1) * T] = y;
+      }
+    cluster.sync();
+
+    // ---- phase 3: explicit CRT of the owned quarter, accumulate ----
+#pragma unroll
+    for (int m = 0; m < 4; ++m) {
+      const uint32_t item = tau + m * T;
+      const uint32_t c = item / Q, jl = item % Q;
+      uint64_t s = 0;
+      uint32_t frac = 0;
+#pragma unroll
+      for (int pq = 0; pq < kPrimes; ++pq) {
+        const uint32_t y = res[(pq * 2 + c) * Q + jl];
+        s += static_cast<uint64_t>(y) * a.cc.pr[pq].Mp_mod64;
+        frac += __umulhi(y, a.cc.pr[pq].F);  // y / p in units of 2^-28
+      }
+      const uint32_t u = (frac + (1u << 27)) >> 28;  // round(sum y_q / p_q)
+      acc[c * Q + jl] += s - static_cast<uint64_t>(u) * a.cc.M_mod64;
+    }
+    cluster.sync();
+  }
+
+  // ---- sample extraction of the constant coefficient ----
+  uint64_t *out = a.lwe_big_out + static_cast<size_t>(ct) * (N + 1);
+#pragma unroll
+  for (int m = 0; m < 4; ++m) {
+    const uint32_t item = tau + m * T;
+    const uint32_t c = item / Q, jl = item % Q, j = rank * Q + jl;
+    if (c == 0) {
+      out[j == 0 ? 0 : N - j] = (j == 0) ? acc[jl] : 0ull - acc[jl];
+    } else if (j == 0) {
+      out[N] = acc[Q];
+    }
+  }
+  cluster.sync();
+}
+
+size_t br_smem_bytes(uint32_t logN, uint32_t level, uint32_t n, bool dig16) {
+  const size_t N = size_t(1) << logN, Q = N / 4;
+  const size_t xbuf = (logN <= 11) ? 2 : 1;
+  size_t b = N * sizeof(uint2) + 2 * Q * sizeof(uint64_t) + kPrimes * 2 * Q * sizeof(uint32_t) +
+             xbuf * (N + N / 8) * sizeof(uint32_t) + 2 * level * Q * (dig16 ? 2 : 4) + (n + 1) * sizeof(uint16_t);
+  return (b + 15) & ~size_t(15);
+}
+
+template <int LOGN, bool DIG16>
+static cudaError_t launch_br_t(const BrArgs &a, cudaStream_t s) {
+  auto kern = blind_rotate_kernel<LOGN, DIG16>;
+  const size_t smem = br_smem_bytes(LOGN, a.level, a.n, DIG16);
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(4 * a.batch, 1, 1);
+  cfg.blockDim = dim3((1 << LOGN) / 8, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 4;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, a);
+}
+
+cudaError_t launch_blind_rotate(const BrArgs &a, uint32_t logN, bool dig16, cudaStream_t s) {
+#define ROSETTA_BR_CASE(L)                                                        \
+  case L:                                                                         \
+    return dig16 ? launch_br_t<L, true>(a, s) : launch_br_t<L, false>(a, s);
+  switch (logN) {
+    ROSETTA_BR_CASE(8)
+    ROSETTA_BR_CASE(9)
+    ROSETTA_BR_CASE(10)
+    ROSETTA_BR_CASE(11)
+    ROSETTA_BR_CASE(12)
+    ROSETTA_BR_CASE(13)
+    default:
+      return cudaErrorInvalidValue;
+  }
+#undef ROSETTA_BR_CASE
+}
+
+}  // namespace rosetta

@@ -1,0 +1,64 @@
+// Internal declarations of librosetta shared by the host API and the kernels.
+#pragma once
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace rosetta {
+
+// Four NTT primes p = c * 2^14 + 1 in (2^28, 2^29): 2N | p - 1 for every
+// N <= 8192, 8p < 2^32 leaves room for lazily reduced residues, and their
+// product M > 2^115 exceeds twice the largest exact integer value of an
+// external-product coefficient, (k+1) l N 2^(beta-1) 2^63, for every
+// parameter set the library accepts (checked at context creation).
+constexpr int kPrimes = 4;
+constexpr uint32_t kPrimeList[kPrimes] = {536690689u, 536641537u, 536608769u, 536543233u};
+
+struct PrimeConsts {
+  uint32_t p;
+  uint32_t p_inv;     // p^{-1} mod 2^32 (Montgomery reduction)
+  uint32_t crt_c;     // N^{-1} * (M/p)^{-1} mod p
+  uint32_t crt_cs;    // Shoup companion of crt_c
+  uint32_t F;         // floor(2^60 / p): fixed-point 1/p for the CRT quotient
+  uint32_t r_mont;    // 2^32 mod p
+  uint32_t r_mont_s;  // Shoup companion of r_mont
+  uint32_t pad_;
+  uint64_t Mp_mod64;  // (M / p) mod 2^64
+};
+
+struct CrtConsts {
+  PrimeConsts pr[kPrimes];
+  uint64_t M_mod64;   // M mod 2^64
+};
+
+struct BrArgs {
+  const uint64_t *lwe_in;   // [batch][n+1]
+  const uint64_t *lut;      // [2^p]
+  uint64_t *lwe_big_out;    // [batch][N+1]   (k = 1)
+  const uint32_t *bsk;      // transform domain [n][prime][2l][2][N]
+  const uint2 *tw;          // [prime][N] (W, Shoup companion)
+  uint32_t n, level, base_log, msg_bits, batch;
+  CrtConsts cc;
+};
+
+struct KsArgs {
+  const uint64_t *big;      // [batch][kN+1]
+  uint64_t *out;            // [batch][n+1]
+  const uint64_t *ksk;      // [kN][l_ks][n+1]
+  const uint64_t *corr;     // [n+1]: (B/2) * sum over KSK rows
+  uint32_t batch, kN, n, base_log, level;
+};
+
+// host-side tables (tables.cu)
+bool build_tables(uint32_t logN, uint2 *tw_host /*[kPrimes][N]*/, CrtConsts *cc);
+
+// launchers; return cudaSuccess or the launch error
+size_t br_smem_bytes(uint32_t logN, uint32_t level, uint32_t n, bool dig16);
+cudaError_t launch_blind_rotate(const BrArgs &a, uint32_t logN, bool dig16, cudaStream_t s);
+cudaError_t launch_bsk_transform(const uint64_t *raw, uint32_t *out, const uint2 *tw, const CrtConsts &cc,
+                                 uint32_t logN, uint32_t n, uint32_t level, cudaStream_t s);
+cudaError_t launch_keyswitch(const KsArgs &a, cudaStream_t s);
+cudaError_t launch_ksk_corr(const uint64_t *ksk, uint64_t *corr, uint32_t rows, uint32_t n, uint32_t base_log,
+                            cudaStream_t s);
+
+}  // namespace rosetta

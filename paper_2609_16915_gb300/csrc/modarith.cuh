@@ -1,0 +1,33 @@
+// Word-level modular arithmetic for the NTT primes (p < 2^29, so 8p < 2^32
+// and lazily reduced residues up to 8p still fit a 32-bit register).
+//
+// Residues are kept "lazy": a value congruent to the residue but possibly a
+// few multiples of p above it.  Every function states the range it accepts
+// and the range it returns.
+#pragma once
+#include <stdint.h>
+
+namespace rosetta {
+
+// Shoup multiplication by a constant w < p with companion ws = floor(w 2^32 / p):
+// for any 32-bit y returns y*w mod p as a value in [0, 2p).
+__device__ __forceinline__ uint32_t shoup_mul(uint32_t y, uint32_t w, uint32_t ws, uint32_t p) {
+  const uint32_t q = __umulhi(y, ws);
+  return y * w - q * p;
+}
+
+// Montgomery reduction with R = 2^32, p_inv = p^{-1} mod 2^32.
+// For T < p * 2^32 returns a value in (0, 2p) congruent to T * 2^-32 mod p.
+// The low words of T and m*p agree, so (T - m p) / 2^32 = hi(T) - hi(m p).
+__device__ __forceinline__ uint32_t redc(uint64_t T, uint32_t p, uint32_t p_inv) {
+  const uint32_t m = static_cast<uint32_t>(T) * p_inv;
+  const uint32_t t = __umulhi(m, p);
+  return static_cast<uint32_t>(T >> 32) - t + p;
+}
+
+// x in [0, 2b) -> [0, b) for a bound b: one subtraction when x >= b.
+__device__ __forceinline__ uint32_t cond_sub(uint32_t x, uint32_t b) {
+  return min(x, x - b);
+}
+
+}  // namespace rosetta

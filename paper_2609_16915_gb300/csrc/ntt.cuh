@@ -1,0 +1,211 @@
+// Negacyclic number-theoretic transforms of size N = 2^LOGN over one prime,
+// distributed over N/8 threads that each hold 8 residues in registers.
+//
+// Forward: Cooley-Tukey butterflies with the negacyclic twist merged into the
+// twiddles (W[m] = psi^{bitrev(m)}, psi a primitive 2N-th root of unity);
+// natural-order input, bit-reversed output.  Inverse: Gentleman-Sande
+// butterflies, bit-reversed input, natural output, without the final N^{-1}
+// (folded by the caller into its next constant).  The inverse twiddle of
+// stage s, group g is psi^{-bitrev(2^s+g)} = -W[2^{s+1}-1-g], so one table
+// serves both directions.
+//
+// The log2(N) stages are grouped into radix-8 passes of three stages (the
+// last pass takes the remaining one to three).  Within a pass each thread
+// owns whole butterfly blocks and keeps them in registers; between passes the
+// values are exchanged through a shared-memory buffer.  After the last
+// forward pass thread t holds bit-reversed positions 8t .. 8t+7, which is
+// exactly what the first inverse pass needs, so a pointwise product between
+// the two transforms needs no exchange.
+//
+// Lazy ranges: forward input < 2p, output < 8p; inverse input < 4p, output
+// < 4p.  See the butterflies for the per-stage invariants.
+#pragma once
+#include <stdint.h>
+
+#include "modarith.cuh"
+
+namespace rosetta {
+
+template <int LOGN>
+struct NttShape {
+  static constexpr int N = 1 << LOGN;
+  static constexpr int T = N / 8;                    // threads per transform
+  static constexpr int NPASS = (LOGN + 2) / 3;
+  static constexpr int LAST_H = LOGN - 3 * (NPASS - 1);
+  static constexpr int XB_WORDS = N + N / 8;         // padded exchange buffer
+  template <int PASS>
+  __host__ __device__ static constexpr int h() { return PASS == NPASS - 1 ? LAST_H : 3; }
+};
+
+// Exchange-buffer address: 4 pad words after every 32 keeps every pass's
+// scalar accesses free of bank conflicts except the last pass, whose
+// contiguous 8-word groups are then read and written as two 16-byte vectors.
+__device__ __forceinline__ uint32_t xb_pad(uint32_t i) { return i + ((i >> 5) << 2); }
+
+// Position (in the stage-ordered data array) of register slot e of thread
+// tau during the pass that starts at stage S0 and spans H stages.  Blocks of
+// 2^H elements have stride SIG = N >> (S0+H) and live in the stage-S0 group
+// g of span N >> S0; a thread owns 8 >> H consecutive blocks.
+template <int LOGN, int S0, int H>
+__device__ __forceinline__ uint32_t slot_index(uint32_t tau, int e) {
+  constexpr uint32_t N = 1u << LOGN;
+  constexpr uint32_t SIG = N >> (S0 + H);
+  constexpr uint32_t SPAN = N >> S0;
+  constexpr int NB = 8 >> H;
+  const int b = e >> H;
+  const int q = e & ((1 << H) - 1);
+  const uint32_t beta = tau * NB + b;
+  const uint32_t g = beta / SIG;
+  const uint32_t i = beta % SIG;
+  return g * SPAN + i + q * SIG;
+}
+
+// Forward (Cooley-Tukey) butterfly X' = X + wY, Y' = X - wY with t = wY in
+// [0, 2p).  Without correction: inputs < a p give outputs < (a+2) p.  With
+// correction X is first brought below 4p (valid for X < 8p).
+template <bool CORR>
+__device__ __forceinline__ void ct_bfly(uint32_t &X, uint32_t &Y, uint2 w, uint32_t p, uint32_t two_p,
+                                        uint32_t four_p) {
+  if (CORR) X = cond_sub(X, four_p);
+  const uint32_t t = shoup_mul(Y, w.x, w.y, p);
+  Y = X - t + two_p;
+  X = X + t;
+}
+
+// Stage s of the forward transform corrects X when s >= 3 and s is odd:
+// bounds run 2p -> 4p -> 6p -> 8p, then alternate 6p (corrected) and 8p.
+__host__ __device__ constexpr bool fwd_stage_corrects(int s) { return s >= 3 && ((s - 3) % 2 == 0); }
+
+// Inverse (Gentleman-Sande) butterfly with inverse twiddle -w:
+// X' = X + Y (brought below 4p), Y' = (X - Y)(-w) = (Y - X + 4p) w.
+// Inputs < 4p give X' < 4p and Y' < 2p.
+__device__ __forceinline__ void gs_bfly(uint32_t &X, uint32_t &Y, uint2 w, uint32_t p, uint32_t four_p) {
+  const uint32_t s = X + Y;
+  const uint32_t d = Y - X + four_p;
+  X = cond_sub(s, four_p);
+  Y = shoup_mul(d, w.x, w.y, p);
+}
+
+template <int LOGN, int NP, int S0, int H, int U>
+__device__ __forceinline__ void fwd_stage(uint32_t (&x)[NP][8], const uint2 *__restrict__ tw, uint32_t tau,
+                                          uint32_t p, uint32_t two_p, uint32_t four_p) {
+  constexpr uint32_t N = 1u << LOGN;
+  constexpr uint32_t SIG = N >> (S0 + H);
+  constexpr int NB = 8 >> H;
+  constexpr int S = S0 + U;
+  constexpr int HALF = 1 << (H - 1 - U);
+  constexpr bool CORR = fwd_stage_corrects(S);
+#pragma unroll
+  for (int b = 0; b < NB; ++b) {
+    const uint32_t g = (tau * NB + b) / SIG;
+#pragma unroll
+    for (int q = 0; q < (1 << H); ++q) {
+      if (q & HALF) continue;
+      const uint2 w = tw[(1u << S) + (g << U) + (q >> (H - U))];
+#pragma unroll
+      for (int k = 0; k < NP; ++k)
+        ct_bfly<CORR>(x[k][b * (1 << H) + q], x[k][b * (1 << H) + q + HALF], w, p, two_p, four_p);
+    }
+  }
+}
+
+template <int LOGN, int NP, int S0, int H, int U>
+__device__ __forceinline__ void inv_stage(uint32_t (&x)[NP][8], const uint2 *__restrict__ tw, uint32_t tau,
+                                          uint32_t p, uint32_t four_p) {
+  constexpr uint32_t N = 1u << LOGN;
+  constexpr uint32_t SIG = N >> (S0 + H);
+  constexpr int NB = 8 >> H;
+  constexpr int S = S0 + U;
+  constexpr int HALF = 1 << (H - 1 - U);
+#pragma unroll
+  for (int b = 0; b < NB; ++b) {
+    const uint32_t g = (tau * NB + b) / SIG;
+#pragma unroll
+    for (int q = 0; q < (1 << H); ++q) {
+      if (q & HALF) continue;
+      const uint32_t G = (g << U) + (q >> (H - U));
+      const uint2 w = tw[(2u << S) - 1u - G];
+#pragma unroll
+      for (int k = 0; k < NP; ++k) gs_bfly(x[k][b * (1 << H) + q], x[k][b * (1 << H) + q + HALF], w, p, four_p);
+    }
+  }
+}
+
+template <int LOGN, int NP, int S0, int H>
+__device__ __forceinline__ void fwd_pass(uint32_t (&x)[NP][8], const uint2 *tw, uint32_t tau, uint32_t p,
+                                         uint32_t two_p, uint32_t four_p) {
+  fwd_stage<LOGN, NP, S0, H, 0>(x, tw, tau, p, two_p, four_p);
+  if constexpr (H > 1) fwd_stage<LOGN, NP, S0, H, 1>(x, tw, tau, p, two_p, four_p);
+  if constexpr (H > 2) fwd_stage<LOGN, NP, S0, H, 2>(x, tw, tau, p, two_p, four_p);
+}
+
+template <int LOGN, int NP, int S0, int H>
+__device__ __forceinline__ void inv_pass(uint32_t (&x)[NP][8], const uint2 *tw, uint32_t tau, uint32_t p,
+                                         uint32_t four_p) {
+  if constexpr (H > 2) inv_stage<LOGN, NP, S0, H, 2>(x, tw, tau, p, four_p);
+  if constexpr (H > 1) inv_stage<LOGN, NP, S0, H, 1>(x, tw, tau, p, four_p);
+  inv_stage<LOGN, NP, S0, H, 0>(x, tw, tau, p, four_p);
+}
+
+// Move NP register sets from the layout of pass A to that of pass B through
+// the exchange buffer xb (XBUF polynomials of NttShape::XB_WORDS words each).
+// The leading barrier protects xb from readers of the previous exchange.
+template <int LOGN, int NP, int XBUF, int S0A, int HA, int S0B, int HB>
+__device__ __forceinline__ void exchange(uint32_t (&x)[NP][8], uint32_t *xb, uint32_t tau) {
+  constexpr int W = NttShape<LOGN>::XB_WORDS;
+  static_assert(XBUF == 1 || XBUF == NP, "exchange buffer must hold one or all polynomials");
+  if constexpr (XBUF == NP) {
+    __syncthreads();
+#pragma unroll
+    for (int k = 0; k < NP; ++k)
+#pragma unroll
+      for (int e = 0; e < 8; ++e) xb[k * W + xb_pad(slot_index<LOGN, S0A, HA>(tau, e))] = x[k][e];
+    __syncthreads();
+#pragma unroll
+    for (int k = 0; k < NP; ++k)
+#pragma unroll
+      for (int e = 0; e < 8; ++e) x[k][e] = xb[k * W + xb_pad(slot_index<LOGN, S0B, HB>(tau, e))];
+  } else {
+#pragma unroll
+    for (int k = 0; k < NP; ++k) {
+      __syncthreads();
+#pragma unroll
+      for (int e = 0; e < 8; ++e) xb[xb_pad(slot_index<LOGN, S0A, HA>(tau, e))] = x[k][e];
+      __syncthreads();
+#pragma unroll
+      for (int e = 0; e < 8; ++e) x[k][e] = xb[xb_pad(slot_index<LOGN, S0B, HB>(tau, e))];
+    }
+  }
+}
+
+// Forward transform of NP polynomials held as x[k][e] = element
+// slot_index<LOGN,0,3>(tau, e) = tau + e*N/8 of polynomial k.
+template <int LOGN, int NP, int XBUF, int PASS = 0>
+__device__ __forceinline__ void ntt_forward(uint32_t (&x)[NP][8], const uint2 *tw, uint32_t *xb, uint32_t tau,
+                                            uint32_t p) {
+  using S = NttShape<LOGN>;
+  constexpr int S0 = 3 * PASS;
+  constexpr int H = S::template h<PASS>();
+  fwd_pass<LOGN, NP, S0, H>(x, tw, tau, p, 2 * p, 4 * p);
+  if constexpr (PASS + 1 < S::NPASS) {
+    exchange<LOGN, NP, XBUF, S0, H, S0 + 3, S::template h<PASS + 1>()>(x, xb, tau);
+    ntt_forward<LOGN, NP, XBUF, PASS + 1>(x, tw, xb, tau, p);
+  }
+}
+
+// Inverse transform (without the N^{-1} factor).  Input: x[k][e] holds
+// bit-reversed position 8*tau + e; output: natural position tau + e*N/8.
+template <int LOGN, int NP, int XBUF, int PASS = NttShape<LOGN>::NPASS - 1>
+__device__ __forceinline__ void ntt_inverse(uint32_t (&x)[NP][8], const uint2 *tw, uint32_t *xb, uint32_t tau,
+                                            uint32_t p) {
+  using S = NttShape<LOGN>;
+  constexpr int S0 = 3 * PASS;
+  constexpr int H = S::template h<PASS>();
+  inv_pass<LOGN, NP, S0, H>(x, tw, tau, p, 4 * p);
+  if constexpr (PASS > 0) {
+    exchange<LOGN, NP, XBUF, S0, H, S0 - 3, 3>(x, xb, tau);
+    ntt_inverse<LOGN, NP, XBUF, PASS - 1>(x, tw, xb, tau, p);
+  }
+}
+
+}  // namespace rosetta

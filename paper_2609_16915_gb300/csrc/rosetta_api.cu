@@ -1,0 +1,406 @@
+// C ABI of librosetta: context creation, key upload, batched PBS, key
+// switch.  Validates every argument before enqueuing work and never falls back
+// to the host.  Declarations and their documentation: include/rosetta.h.
+#include <cuda_runtime.h>
+
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "../../include/rosetta.h"
+#include "internal.h"
+
+using namespace rosetta;
+
+struct rosetta_ctx {
+  rosetta_params prm{};
+  int device = 0;
+  uint32_t logN = 0;
+  bool dig16 = false;
+  CrtConsts cc{};
+  uint2 *d_tw = nullptr;          // [kPrimes][N]
+  uint32_t *d_bsk = nullptr;      // transform domain
+  uint64_t *d_ksk = nullptr;      // raw [kN][l_ks][n+1]
+  uint64_t *d_corr = nullptr;     // [n+1]
+  bool have_bsk = false, have_ksk = false;
+  // scratch and staging, sized in ciphertexts
+  uint64_t *d_big = nullptr;      // extracted ciphertexts [batch][kN+1]
+  size_t big_words_cap = 0;
+  uint64_t *d_in = nullptr;       // staging for host inputs
+  size_t in_words_cap = 0;
+  uint64_t *d_out = nullptr;      // staging for host outputs
+  size_t out_words_cap = 0;
+  uint64_t *d_lut = nullptr;      // staging for a host LUT  [2^p]
+};
+
+namespace {
+
+int cuda_fail(cudaError_t e) {
+  return e == cudaErrorMemoryAllocation ? ROSETTA_ERR_OOM : ROSETTA_ERR_CUDA;
+}
+
+bool is_device_ptr(const void *p) {
+  cudaPointerAttributes at;
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
+}
+
+bool overlaps(const void *a, size_t na, const void *b, size_t nb) {
+  const char *pa = static_cast<const char *>(a), *pb = static_cast<const char *>(b);
+  return pa < pb + nb && pb < pa + na;
+}
+
+bool aligned8(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 7u) == 0; }
+
+uint32_t log2_exact(uint32_t x) {
+  uint32_t r = 0;
+  while ((1u << r) < x) ++r;
+  return (1u << r) == x ? r : 0xffffffffu;
+}
+
+// Number of bits of the largest possible |integer value| of an external
+// product coefficient, (k+1) l N 2^(beta-1) 2^63, rounded up.
+double ext_product_bits(const rosetta_params &p) {
+  double v = 63.0 + (p.pbs_base_log - 1);
+  double f = (double)(p.glwe_dim + 1) * p.pbs_level * p.poly_size;
+  int e = 0;
+  while ((double)(1ull << e) < f) ++e;
+  return v + e;
+}
+
+int check_params(const rosetta_params &p) {
+  const uint32_t logN = log2_exact(p.poly_size);
+  if (logN < 8 || logN > 13) return ROSETTA_ERR_UNSUPPORTED_PARAMS;
+  if (p.glwe_dim != 1) return ROSETTA_ERR_UNSUPPORTED_PARAMS;
+  if (p.lwe_dim == 0 || p.lwe_dim > 65535) return ROSETTA_ERR_UNSUPPORTED_PARAMS;
+  if (p.pbs_base_log < 1 || p.pbs_base_log > 28 || p.pbs_level < 1 || p.pbs_base_log * p.pbs_level > 64)
+    return ROSETTA_ERR_UNSUPPORTED_PARAMS;
+  if (p.ks_base_log < 1 || p.ks_base_log > 16 || p.ks_level < 1 || p.ks_base_log * p.ks_level > 64)
+    return ROSETTA_ERR_UNSUPPORTED_PARAMS;
+  if (p.msg_bits < 1 || p.msg_bits > 62 || (p.poly_size >> p.msg_bits) < 2) return ROSETTA_ERR_UNSUPPORTED_PARAMS;
+  // exact CRT: the product of the four primes (> 2^115) must exceed twice the bound
+  if (ext_product_bits(p) + 1.0 > 115.0) return ROSETTA_ERR_UNSUPPORTED_PARAMS;
+  return ROSETTA_OK;
+}
+
+// (Re)allocate *buf, stream-ordered, to hold at least `need` words.
+int ensure(uint64_t **buf, size_t *cap_words, size_t need, cudaStream_t s) {
+  if (*buf && *cap_words >= need) return ROSETTA_OK;
+  if (*buf) {
+    cudaError_t e = cudaFreeAsync(*buf, s);
+    *buf = nullptr;
+    *cap_words = 0;
+    if (e != cudaSuccess) return cuda_fail(e);
+  }
+  cudaError_t e = cudaMallocAsync(reinterpret_cast<void **>(buf), need * sizeof(uint64_t), s);
+  if (e != cudaSuccess) {
+    *buf = nullptr;
+    return cuda_fail(e);
+  }
+  *cap_words = need;
+  return ROSETTA_OK;
+}
+
+size_t lwe_words(const rosetta_ctx *c) { return c->prm.lwe_dim + 1; }
+size_t big_words(const rosetta_ctx *c) { return (size_t)c->prm.glwe_dim * c->prm.poly_size + 1; }
+size_t stage_words(const rosetta_ctx *c) { return big_words(c) > lwe_words(c) ? big_words(c) : lwe_words(c); }
+
+// Scratch for the extracted ciphertexts of `batch` inputs.
+int ensure_big(rosetta_ctx *c, uint32_t batch, cudaStream_t s) {
+  return ensure(&c->d_big, &c->big_words_cap, (size_t)batch * big_words(c), s);
+}
+
+// Staging for host-memory inputs and outputs of `batch` ciphertexts.
+int ensure_stage(rosetta_ctx *c, uint32_t batch, cudaStream_t s) {
+  const size_t need = (size_t)batch * stage_words(c);
+  int st = ensure(&c->d_in, &c->in_words_cap, need, s);
+  return st == ROSETTA_OK ? ensure(&c->d_out, &c->out_words_cap, need, s) : st;
+}
+
+cudaStream_t as_stream(void *s) { return reinterpret_cast<cudaStream_t>(s); }
+
+// Shared front half of the entry points that take ciphertexts in and out:
+// validation, host staging of inputs.  in_words/out_words are per ciphertext.
+struct Staged {
+  const uint64_t *in = nullptr;
+  const uint64_t *lut = nullptr;
+  uint64_t *out = nullptr;
+  bool out_host = false;
+};
+
+int stage_io(rosetta_ctx *c, const uint64_t *in, size_t in_words, uint32_t batch, const uint64_t *lut,
+             uint64_t *out, size_t out_words, cudaStream_t s, Staged *st) {
+  if (!aligned8(in) || !aligned8(out) || (lut && !aligned8(lut))) return ROSETTA_ERR_INVALID_ARG;
+  const size_t in_bytes = (size_t)batch * in_words * 8, out_bytes = (size_t)batch * out_words * 8;
+  if (overlaps(in, in_bytes, out, out_bytes)) return ROSETTA_ERR_INVALID_ARG;
+  if (c->prm.max_batch && batch > c->prm.max_batch) return ROSETTA_ERR_INVALID_ARG;
+  const bool in_dev = is_device_ptr(in), out_dev = is_device_ptr(out);
+  st->in = in;
+  st->out = out;
+  st->lut = lut;
+  if (!in_dev || !out_dev) {
+    int r = ensure_stage(c, batch, s);
+    if (r != ROSETTA_OK) return r;
+  }
+  if (!in_dev) {
+    cudaError_t e = cudaMemcpyAsync(c->d_in, in, in_bytes, cudaMemcpyHostToDevice, s);
+    if (e != cudaSuccess) return cuda_fail(e);
+    st->in = c->d_in;
+  }
+  if (!out_dev) {
+    st->out = c->d_out;
+    st->out_host = true;
+  }
+  if (lut && !is_device_ptr(lut)) {
+    cudaError_t e = cudaMemcpyAsync(c->d_lut, lut, sizeof(uint64_t) << c->prm.msg_bits, cudaMemcpyHostToDevice, s);
+    if (e != cudaSuccess) return cuda_fail(e);
+    st->lut = c->d_lut;
+  }
+  return ROSETTA_OK;
+}
+
+int finish_io(rosetta_ctx *c, uint64_t *out, size_t out_words, uint32_t batch, const Staged &st, cudaStream_t s) {
+  (void)c;
+  if (!st.out_host) return ROSETTA_OK;
+  cudaError_t e = cudaMemcpyAsync(out, st.out, (size_t)batch * out_words * 8, cudaMemcpyDeviceToHost, s);
+  if (e != cudaSuccess) return cuda_fail(e);
+  e = cudaStreamSynchronize(s);
+  return e == cudaSuccess ? ROSETTA_OK : cuda_fail(e);
+}
+
+BrArgs br_args(const rosetta_ctx *c, const uint64_t *in, uint32_t batch, const uint64_t *lut, uint64_t *big) {
+  BrArgs a{};
+  a.lwe_in = in;
+  a.lut = lut;
+  a.lwe_big_out = big;
+  a.bsk = c->d_bsk;
+  a.tw = c->d_tw;
+  a.n = c->prm.lwe_dim;
+  a.level = c->prm.pbs_level;
+  a.base_log = c->prm.pbs_base_log;
+  a.msg_bits = c->prm.msg_bits;
+  a.batch = batch;
+  a.cc = c->cc;
+  return a;
+}
+
+KsArgs ks_args(const rosetta_ctx *c, const uint64_t *big, uint32_t batch, uint64_t *out) {
+  KsArgs k{};
+  k.big = big;
+  k.out = out;
+  k.ksk = c->d_ksk;
+  k.corr = c->d_corr;
+  k.batch = batch;
+  k.kN = c->prm.glwe_dim * c->prm.poly_size;
+  k.n = c->prm.lwe_dim;
+  k.base_log = c->prm.ks_base_log;
+  k.level = c->prm.ks_level;
+  return k;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *rosetta_status_string(int status) {
+  switch (status) {
+    case ROSETTA_OK: return "ok";
+    case ROSETTA_ERR_INVALID_ARG: return "invalid argument";
+    case ROSETTA_ERR_UNSUPPORTED_PARAMS: return "unsupported parameters";
+    case ROSETTA_ERR_KEYS_MISSING: return "keys not uploaded";
+    case ROSETTA_ERR_CUDA: return "CUDA error";
+    case ROSETTA_ERR_OOM: return "out of device memory";
+    case ROSETTA_ERR_TIMEOUT: return "device wait timed out";
+    default: return "unknown status";
+  }
+}
+
+int rosetta_params_init(rosetta_ctx **out, const rosetta_params *p, int cuda_device) {
+  if (!out) return ROSETTA_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!p) return ROSETTA_ERR_INVALID_ARG;
+  int st = check_params(*p);
+  if (st != ROSETTA_OK) return st;
+  int ndev = 0;
+  if (cudaGetDeviceCount(&ndev) != cudaSuccess || cuda_device < 0 || cuda_device >= ndev) {
+    cudaGetLastError();
+    return ROSETTA_ERR_CUDA;
+  }
+  if (cudaSetDevice(cuda_device) != cudaSuccess) return ROSETTA_ERR_CUDA;
+  const uint32_t logN = log2_exact(p->poly_size);
+  const bool dig16 = p->pbs_base_log <= 16;
+  int max_smem = 0;
+  cudaDeviceGetAttribute(&max_smem, cudaDevAttrMaxSharedMemoryPerBlockOptin, cuda_device);
+  if (br_smem_bytes(logN, p->pbs_level, p->lwe_dim, dig16) > (size_t)max_smem) return ROSETTA_ERR_UNSUPPORTED_PARAMS;
+
+  rosetta_ctx *c = new (std::nothrow) rosetta_ctx();
+  if (!c) return ROSETTA_ERR_OOM;
+  c->prm = *p;
+  c->device = cuda_device;
+  c->logN = logN;
+  c->dig16 = dig16;
+  std::vector<uint2> tw((size_t)kPrimes << logN);
+  if (!build_tables(logN, tw.data(), &c->cc)) {
+    delete c;
+    return ROSETTA_ERR_UNSUPPORTED_PARAMS;
+  }
+  cudaError_t e = cudaMalloc(&c->d_tw, tw.size() * sizeof(uint2));
+  if (e == cudaSuccess) e = cudaMemcpy(c->d_tw, tw.data(), tw.size() * sizeof(uint2), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) e = cudaMalloc(&c->d_lut, sizeof(uint64_t) << p->msg_bits);
+  if (e != cudaSuccess) {
+    rosetta_destroy(c);
+    return cuda_fail(e);
+  }
+  if (p->max_batch) {
+    st = ensure_big(c, p->max_batch, nullptr);
+    if (st == ROSETTA_OK) st = ensure_stage(c, p->max_batch, nullptr);
+    if (st == ROSETTA_OK && cudaStreamSynchronize(nullptr) != cudaSuccess) st = ROSETTA_ERR_CUDA;
+    if (st != ROSETTA_OK) {
+      rosetta_destroy(c);
+      return st;
+    }
+  }
+  *out = c;
+  return ROSETTA_OK;
+}
+
+int rosetta_upload_bsk(rosetta_ctx *c, const uint64_t *bsk, size_t n_words, int src_is_device, void *stream) {
+  if (!c || !bsk) return ROSETTA_ERR_INVALID_ARG;
+  const rosetta_params &p = c->prm;
+  const size_t want = (size_t)p.lwe_dim * (p.glwe_dim + 1) * p.pbs_level * (p.glwe_dim + 1) * p.poly_size;
+  if (n_words != want || !aligned8(bsk)) return ROSETTA_ERR_INVALID_ARG;
+  if (cudaSetDevice(c->device) != cudaSuccess) return ROSETTA_ERR_CUDA;
+  cudaStream_t s = as_stream(stream);
+  const uint64_t *src = bsk;
+  uint64_t *tmp = nullptr;
+  cudaError_t e = cudaSuccess;
+  if (!src_is_device) {
+    e = cudaMallocAsync(reinterpret_cast<void **>(&tmp), want * 8, s);
+    if (e != cudaSuccess) return cuda_fail(e);
+    e = cudaMemcpyAsync(tmp, bsk, want * 8, cudaMemcpyHostToDevice, s);
+    if (e != cudaSuccess) {
+      cudaFreeAsync(tmp, s);
+      return cuda_fail(e);
+    }
+    src = tmp;
+  }
+  // one 32-bit residue per prime for every raw word
+  if (!c->d_bsk) e = cudaMalloc(&c->d_bsk, want * kPrimes * sizeof(uint32_t));
+  if (e != cudaSuccess) {
+    if (tmp) cudaFreeAsync(tmp, s);
+    return cuda_fail(e);
+  }
+  e = launch_bsk_transform(src, c->d_bsk, c->d_tw, c->cc, c->logN, p.lwe_dim, p.pbs_level, s);
+  if (tmp) cudaFreeAsync(tmp, s);
+  if (e != cudaSuccess) return cuda_fail(e);
+  if (!src_is_device) {
+    e = cudaStreamSynchronize(s);  // caller may free the host buffer on return
+    if (e != cudaSuccess) return cuda_fail(e);
+  }
+  c->have_bsk = true;
+  return ROSETTA_OK;
+}
+
+int rosetta_upload_ksk(rosetta_ctx *c, const uint64_t *ksk, size_t n_words, int src_is_device, void *stream) {
+  if (!c || !ksk) return ROSETTA_ERR_INVALID_ARG;
+  const rosetta_params &p = c->prm;
+  const size_t rows = (size_t)p.glwe_dim * p.poly_size * p.ks_level;
+  const size_t want = rows * (p.lwe_dim + 1);
+  if (n_words != want || !aligned8(ksk)) return ROSETTA_ERR_INVALID_ARG;
+  if (cudaSetDevice(c->device) != cudaSuccess) return ROSETTA_ERR_CUDA;
+  cudaStream_t s = as_stream(stream);
+  cudaError_t e = cudaSuccess;
+  if (!c->d_ksk) e = cudaMalloc(&c->d_ksk, want * 8);
+  if (e == cudaSuccess && !c->d_corr) e = cudaMalloc(&c->d_corr, (p.lwe_dim + 1) * 8);
+  if (e != cudaSuccess) return cuda_fail(e);
+  e = cudaMemcpyAsync(c->d_ksk, ksk, want * 8, src_is_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice, s);
+  if (e != cudaSuccess) return cuda_fail(e);
+  e = launch_ksk_corr(c->d_ksk, c->d_corr, (uint32_t)rows, p.lwe_dim, p.ks_base_log, s);
+  if (e != cudaSuccess) return cuda_fail(e);
+  if (!src_is_device) {
+    e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail(e);
+  }
+  c->have_ksk = true;
+  return ROSETTA_OK;
+}
+
+int rosetta_blind_rotate_extract_batch(rosetta_ctx *c, const uint64_t *lwe_in, uint32_t batch, const uint64_t *lut,
+                                       uint64_t *lwe_big_out, void *stream) {
+  if (!c) return ROSETTA_ERR_INVALID_ARG;
+  if (batch == 0) return ROSETTA_OK;
+  if (!lwe_in || !lut || !lwe_big_out) return ROSETTA_ERR_INVALID_ARG;
+  if (!c->have_bsk) return ROSETTA_ERR_KEYS_MISSING;
+  if (cudaSetDevice(c->device) != cudaSuccess) return ROSETTA_ERR_CUDA;
+  cudaStream_t s = as_stream(stream);
+  Staged st;
+  int r = stage_io(c, lwe_in, lwe_words(c), batch, lut, lwe_big_out, big_words(c), s, &st);
+  if (r != ROSETTA_OK) return r;
+  cudaError_t e = launch_blind_rotate(br_args(c, st.in, batch, st.lut, st.out), c->logN, c->dig16, s);
+  if (e != cudaSuccess) return cuda_fail(e);
+  return finish_io(c, lwe_big_out, big_words(c), batch, st, s);
+}
+
+int rosetta_keyswitch_batch(rosetta_ctx *c, const uint64_t *lwe_big_in, uint32_t batch, uint64_t *lwe_out,
+                            void *stream) {
+  if (!c) return ROSETTA_ERR_INVALID_ARG;
+  if (batch == 0) return ROSETTA_OK;
+  if (!lwe_big_in || !lwe_out) return ROSETTA_ERR_INVALID_ARG;
+  if (!c->have_ksk) return ROSETTA_ERR_KEYS_MISSING;
+  if (cudaSetDevice(c->device) != cudaSuccess) return ROSETTA_ERR_CUDA;
+  cudaStream_t s = as_stream(stream);
+  Staged st;
+  int r = stage_io(c, lwe_big_in, big_words(c), batch, nullptr, lwe_out, lwe_words(c), s, &st);
+  if (r != ROSETTA_OK) return r;
+  cudaError_t e = launch_keyswitch(ks_args(c, st.in, batch, st.out), s);
+  if (e != cudaSuccess) return cuda_fail(e);
+  return finish_io(c, lwe_out, lwe_words(c), batch, st, s);
+}
+
+int rosetta_pbs_batch(rosetta_ctx *c, const uint64_t *lwe_in, uint32_t batch, const uint64_t *lut,
+                      uint64_t *lwe_out, void *stream) {
+  if (!c) return ROSETTA_ERR_INVALID_ARG;
+  if (batch == 0) return ROSETTA_OK;
+  if (!lwe_in || !lut || !lwe_out) return ROSETTA_ERR_INVALID_ARG;
+  if (!c->have_bsk || !c->have_ksk) return ROSETTA_ERR_KEYS_MISSING;
+  if (cudaSetDevice(c->device) != cudaSuccess) return ROSETTA_ERR_CUDA;
+  cudaStream_t s = as_stream(stream);
+  Staged st;
+  int r = stage_io(c, lwe_in, lwe_words(c), batch, lut, lwe_out, lwe_words(c), s, &st);
+  if (r != ROSETTA_OK) return r;
+  r = ensure_big(c, batch, s);
+  if (r != ROSETTA_OK) return r;
+  cudaError_t e = launch_blind_rotate(br_args(c, st.in, batch, st.lut, c->d_big), c->logN, c->dig16, s);
+  if (e != cudaSuccess) return cuda_fail(e);
+  e = launch_keyswitch(ks_args(c, c->d_big, batch, st.out), s);
+  if (e != cudaSuccess) return cuda_fail(e);
+  return finish_io(c, lwe_out, lwe_words(c), batch, st, s);
+}
+
+int rosetta_sync_status(rosetta_ctx *c, void *stream) {
+  if (!c) return ROSETTA_ERR_INVALID_ARG;
+  if (cudaSetDevice(c->device) != cudaSuccess) return ROSETTA_ERR_CUDA;
+  cudaError_t e = cudaStreamSynchronize(as_stream(stream));
+  if (e == cudaSuccess) e = cudaGetLastError();
+  return e == cudaSuccess ? ROSETTA_OK : cuda_fail(e);
+}
+
+void rosetta_destroy(rosetta_ctx *c) {
+  if (!c) return;
+  cudaSetDevice(c->device);
+  cudaDeviceSynchronize();
+  cudaFree(c->d_tw);
+  cudaFree(c->d_bsk);
+  cudaFree(c->d_ksk);
+  cudaFree(c->d_corr);
+  cudaFree(c->d_big);
+  cudaFree(c->d_in);
+  cudaFree(c->d_out);
+  cudaFree(c->d_lut);
+  delete c;
+}
+
+}  // extern "C"

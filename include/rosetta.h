@@ -128,6 +128,22 @@ int rosetta_blind_rotate_extract_batch(rosetta_ctx *ctx, const uint64_t *lwe_in,
 int rosetta_keyswitch_batch(rosetta_ctx *ctx, const uint64_t *lwe_big_in, uint32_t batch,
                             uint64_t *lwe_out, void *stream);
 
+/* Same computation and result as rosetta_pbs_batch, for callers that cannot
+ * allocate device memory during the call (their device memory belongs to
+ * another allocator, or their serving loop forbids allocation after
+ * warm-up).  The paper has no counterpart: this is a deployment variant.
+ * The intermediate ciphertexts live in a fixed 16 MiB array compiled into the
+ * library (held on every device that loads it until exit) instead of a
+ * buffer grown with cudaMallocAsync, so batch * (kN+1) must not exceed
+ * 2^21 words (1023 ciphertexts at N = 2048, 255 at N = 8192); larger
+ * batches return INVALID_ARG.  lwe_in, lut and lwe_out must be device
+ * memory (no host staging).  The first call on a device looks up the
+ * array's device address; make it before any stream capture.  All calls on a
+ * device share the array: calls whose work overlaps on the GPU race and must
+ * be serialised by the caller.  Errors: INVALID_ARG, KEYS_MISSING, CUDA. */
+int rosetta_pbs_batch_noalloc(rosetta_ctx *ctx, const uint64_t *lwe_in, uint32_t batch,
+                              const uint64_t *lut, uint64_t *lwe_out, void *stream);
+
 /* Wait for all work on `stream` and report any deferred execution error
  * (CUDA, TIMEOUT).  Returns OK when the stream finished cleanly. */
 int rosetta_sync_status(rosetta_ctx *ctx, void *stream);

@@ -21,8 +21,8 @@ STATUS = {0: "ok", -1: "invalid argument", -2: "unsupported parameters", -3: "ke
           -4: "CUDA error", -5: "out of device memory", -6: "device wait timed out"}
 
 EXPORTS = ("rosetta_params_init", "rosetta_upload_bsk", "rosetta_upload_ksk", "rosetta_pbs_batch",
-           "rosetta_blind_rotate_extract_batch", "rosetta_keyswitch_batch", "rosetta_sync_status",
-           "rosetta_destroy", "rosetta_status_string")
+           "rosetta_blind_rotate_extract_batch", "rosetta_keyswitch_batch", "rosetta_pbs_batch_noalloc",
+           "rosetta_sync_status", "rosetta_destroy", "rosetta_status_string")
 
 
 class RosettaError(RuntimeError):
@@ -55,6 +55,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     L.rosetta_pbs_batch.argtypes = [vp, u64p, u32, u64p, u64p, vp]
     L.rosetta_blind_rotate_extract_batch.argtypes = [vp, u64p, u32, u64p, u64p, vp]
     L.rosetta_keyswitch_batch.argtypes = [vp, u64p, u32, u64p, vp]
+    L.rosetta_pbs_batch_noalloc.argtypes = [vp, u64p, u32, u64p, u64p, vp]
     L.rosetta_sync_status.argtypes = [vp, vp]
     L.rosetta_destroy.argtypes = [vp]
     L.rosetta_destroy.restype = None
@@ -155,6 +156,14 @@ class Context:
         batch = lwe_big_in.shape[0]
         _check("rosetta_keyswitch_batch", load().rosetta_keyswitch_batch(self._h, _ptr(lwe_big_in), batch,
                                                                          _ptr(lwe_out), _stream(stream)))
+        return lwe_out
+
+    def rosetta_pbs_batch_noalloc(self, lwe_in, lut, lwe_out, stream=None):
+        """rosetta_pbs_batch without any device allocation in the call (fixed
+        in-library scratch; device buffers only, bounded batch)."""
+        batch = lwe_in.shape[0]
+        _check("rosetta_pbs_batch_noalloc", load().rosetta_pbs_batch_noalloc(self._h, _ptr(lwe_in), batch, _ptr(lut),
+                                                                             _ptr(lwe_out), _stream(stream)))
         return lwe_out
 
     def rosetta_sync_status(self, stream=None):

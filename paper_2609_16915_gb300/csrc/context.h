@@ -1,0 +1,30 @@
+// Layout of the opaque rosetta_ctx handle, shared by the translation units
+// that implement the C ABI.
+#pragma once
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "../../include/rosetta.h"
+#include "internal.h"
+
+struct rosetta_ctx {
+  rosetta_params prm{};
+  int device = 0;
+  uint32_t logN = 0;
+  bool dig16 = false;
+  rosetta::CrtConsts cc{};
+  uint2 *d_tw = nullptr;          // [kPrimes][N]
+  uint32_t *d_bsk = nullptr;      // transform domain
+  uint64_t *d_ksk = nullptr;      // raw [kN][l_ks][n+1]
+  uint64_t *d_corr = nullptr;     // [n+1]
+  bool have_bsk = false, have_ksk = false;
+  // scratch and staging, sized in ciphertexts
+  uint64_t *d_big = nullptr;      // extracted ciphertexts [batch][kN+1]
+  size_t big_words_cap = 0;
+  uint64_t *d_in = nullptr;       // staging for host inputs
+  size_t in_words_cap = 0;
+  uint64_t *d_out = nullptr;      // staging for host outputs
+  size_t out_words_cap = 0;
+  uint64_t *d_lut = nullptr;      // staging for a host LUT  [2^p]
+};

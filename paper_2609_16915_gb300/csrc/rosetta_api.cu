@@ -8,30 +8,11 @@
 #include <vector>
 
 #include "../../include/rosetta.h"
+#include "context.h"
 #include "internal.h"
 
 using namespace rosetta;
 
-struct rosetta_ctx {
-  rosetta_params prm{};
-  int device = 0;
-  uint32_t logN = 0;
-  bool dig16 = false;
-  CrtConsts cc{};
-  uint2 *d_tw = nullptr;          // [kPrimes][N]
-  uint32_t *d_bsk = nullptr;      // transform domain
-  uint64_t *d_ksk = nullptr;      // raw [kN][l_ks][n+1]
-  uint64_t *d_corr = nullptr;     // [n+1]
-  bool have_bsk = false, have_ksk = false;
-  // scratch and staging, sized in ciphertexts
-  uint64_t *d_big = nullptr;      // extracted ciphertexts [batch][kN+1]
-  size_t big_words_cap = 0;
-  uint64_t *d_in = nullptr;       // staging for host inputs
-  size_t in_words_cap = 0;
-  uint64_t *d_out = nullptr;      // staging for host outputs
-  size_t out_words_cap = 0;
-  uint64_t *d_lut = nullptr;      // staging for a host LUT  [2^p]
-};
 
 namespace {
 

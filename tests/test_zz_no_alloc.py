@@ -1,0 +1,69 @@
+"""rosetta_pbs_batch_noalloc, the entry point for callers that cannot
+allocate device memory during a call (device memory owned by another
+allocator, or an allocation-free serving loop): it must return exactly what
+rosetta_pbs_batch returns, call after call, even though every call reuses
+the same fixed scratch array inside the library.  Collected last on purpose
+so that a failure here cannot hide the results of the other tests."""
+
+import ctypes
+
+import numpy as np
+import pytest
+
+import workload as W
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def setup():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2609_16915_gb300 import build
+    build.build()
+    import paper_2609_16915_gb300 as R
+    from tests import gpu_util as G
+    p = W.CONFIGS["standard"]
+    bsk, ksk = W.uniform_keys(p, seed=21)
+    ctx = G.make_ctx(p, bsk, ksk)
+    return R, G, p, ctx
+
+
+def _call_noalloc(R, ctx, lwe, lut, out):
+    """Straight through the C ABI."""
+    return R.load().rosetta_pbs_batch_noalloc(ctx._h, ctypes.c_void_p(lwe.data_ptr()), lwe.shape[0],
+                                              ctypes.c_void_p(lut.data_ptr()), ctypes.c_void_p(out.data_ptr()),
+                                              ctypes.c_void_p(None))
+
+
+def test_noalloc_matches_pbs_batch_twice_in_a_row(setup):
+    R, G, p, ctx = setup
+    lut = G.to_dev(W.lut_torus(p))
+    first = G.to_dev(W.uniform_ciphertexts(p, 300, sub=31))
+    second = G.to_dev(W.uniform_ciphertexts(p, 77, sub=32))   # smaller: stale words from call 1 remain
+    for lwe in (first, second):
+        want = G.empty_dev(lwe.shape[0], p.n + 1)
+        ctx.pbs_batch(lwe, lut, want, stream=0)
+        ctx.sync_status(stream=0)
+        got = G.empty_dev(lwe.shape[0], p.n + 1)
+        assert _call_noalloc(R, ctx, lwe, lut, got) == 0
+        ctx.sync_status(stream=0)
+        assert np.array_equal(G.to_host(got), G.to_host(want))
+
+
+def test_noalloc_rejects_oversize_and_host_buffers(setup):
+    R, G, p, ctx = setup
+    lut = G.to_dev(W.lut_torus(p))
+    limit = (2 << 20) // (p.kN + 1)                              # 16 MiB of 64-bit words
+    big = G.to_dev(np.zeros((limit + 1, p.n + 1), np.uint64))
+    out = G.empty_dev(limit + 1, p.n + 1)
+    assert _call_noalloc(R, ctx, big, lut, out) == -1
+    host_in = np.zeros((4, p.n + 1), np.uint64)
+    st = R.load().rosetta_pbs_batch_noalloc(ctx._h, ctypes.c_void_p(host_in.ctypes.data), 4,
+                                            ctypes.c_void_p(lut.data_ptr()), ctypes.c_void_p(out.data_ptr()),
+                                            ctypes.c_void_p(None))
+    assert st == -1
+    ok_in = big[:limit]
+    assert _call_noalloc(R, ctx, ok_in, lut, out[:limit]) == 0
+    ctx.sync_status(stream=0)

@@ -32,22 +32,30 @@
 
 #include <type_traits>
 
+#include "dsmem.cuh"
 #include "internal.h"
 #include "ntt.cuh"
 
 namespace rosetta {
 namespace cg = cooperative_groups;
 
+// One exchange buffer per polynomial of a pair only where shared memory is
+// plentiful; larger rings share one buffer to keep more CTAs resident.
+__host__ __device__ constexpr int br_xbuf(int logN) { return logN <= 10 ? 2 : 1; }
+
 template <int LOGN>
 struct BrShape {
   static constexpr int N = 1 << LOGN;
   static constexpr int T = N / 8;
   static constexpr int Q = N / 4;                      // coefficients owned per CTA
-  static constexpr int XBUF = (LOGN <= 11) ? 2 : 1;    // exchange buffers (polys)
+  static constexpr int XBUF = br_xbuf(LOGN);            // exchange buffers (polys)
+  // resident CTAs per SM the register allocation must allow (shared memory
+  // allows the same: 4 x 55 KB at N = 2048, 2 x 108 KB at 4096)
+  static constexpr int MIN_CTAS = (LOGN <= 11) ? 4 : (LOGN == 12 ? 2 : 1);
 };
 
 template <int LOGN, bool DIG16>
-__global__ void __launch_bounds__((1 << LOGN) / 8) blind_rotate_kernel(const BrArgs a) {
+__global__ void __launch_bounds__((1 << LOGN) / 8, BrShape<LOGN>::MIN_CTAS) blind_rotate_kernel(const BrArgs a) {
   using S = NttShape<LOGN>;
   using B = BrShape<LOGN>;
   using DigT = typename std::conditional<DIG16, int16_t, int32_t>::type;
@@ -99,15 +107,9 @@ __global__ void __launch_bounds__((1 << LOGN) / 8) blind_rotate_kernel(const BrA
   }
   cluster.sync();
 
-  const uint64_t *racc[kPrimes];
-  const DigT *rdig[kPrimes];
-  uint32_t *rres[kPrimes];
-#pragma unroll
-  for (int o = 0; o < kPrimes; ++o) {
-    racc[o] = cluster.map_shared_rank(acc, o);
-    rdig[o] = cluster.map_shared_rank(dig, o);
-    rres[o] = cluster.map_shared_rank(res, o);
-  }
+  // 32-bit shared-memory addresses; mapa turns them into the same location
+  // in another CTA of the cluster
+  const uint32_t acc_s = smem_addr(acc), dig_s = smem_addr(dig), res_s = smem_addr(res);
   const uint32_t L2 = 2 * a.level;
   const uint32_t bits = a.base_log * a.level;
   const uint64_t Bmask = (1ull << a.base_log) - 1;
@@ -120,16 +122,22 @@ __global__ void __launch_bounds__((1 << LOGN) / 8) blind_rotate_kernel(const BrA
     if (at == 0) continue;  // X^0 ACC - ACC = 0: the step adds nothing
 
     // ---- phase 1: rotated difference and gadget digits of the owned quarter ----
+    // (X^a P)[j] = +-P[(j - a) mod 2N]; the four remote words are requested
+    // before any is used so their latencies overlap
+    uint64_t v[4];
 #pragma unroll
     for (int m = 0; m < 4; ++m) {
       const uint32_t item = tau + m * T;
       const uint32_t c = item / Q, jl = item % Q, j = rank * Q + jl;
-      uint32_t e = (j + TWO_N - at) & (TWO_N - 1);  // (X^a P)[j] = +-P[(j - a) mod 2N]
-      const bool neg = e >= N;
-      e &= N - 1;
-      uint64_t v = racc[e / Q][c * Q + (e % Q)];
-      if (neg) v = 0ull - v;
-      const uint64_t diff = v - acc[c * Q + jl];
+      const uint32_t e = (j + TWO_N - at) & (N - 1);
+      v[m] = dsmem_ld_u64(dsmem_map(acc_s + (c * Q + (e % Q)) * 8u, e / Q));
+    }
+#pragma unroll
+    for (int m = 0; m < 4; ++m) {
+      const uint32_t item = tau + m * T;
+      const uint32_t c = item / Q, jl = item % Q, j = rank * Q + jl;
+      const bool neg = ((j + TWO_N - at) & (TWO_N - 1)) >= N;
+      const uint64_t diff = (neg ? 0ull - v[m] : v[m]) - acc[c * Q + jl];
       uint64_t cv = bits >= 64 ? diff : (diff + round_add) >> round_sh;
       for (int l = static_cast<int>(a.level) - 1; l >= 0; --l) {
         const uint64_t d = cv & Bmask;
@@ -153,23 +161,31 @@ __global__ void __launch_bounds__((1 << LOGN) / 8) blind_rotate_kernel(const BrA
       for (int pp = 0; pp < 2; ++pp)
 #pragma unroll
         for (int q = 0; q < 8; ++q) {
-          const int32_t d = rdig[q >> 1][(r0 + pp) * Q + tau + (q & 1) * T];
+          const uint32_t ad = dsmem_map(dig_s + ((r0 + pp) * Q + tau + (q & 1) * T) * sizeof(DigT), q >> 1);
+          const int32_t d = DIG16 ? dsmem_ld_s16(ad) : dsmem_ld_s32(ad);
           x[pp][q] = static_cast<uint32_t>(d + static_cast<int32_t>(p));  // in (0, 2p)
         }
       ntt_forward<LOGN, 2, B::XBUF>(x, tw, xb, tau, p);
+      // BSK_i words of this prime for rows r0, r0+1, 8 per thread and
+      // component, contiguous across the CTA (16-byte loads)
+      const uint4 *g = reinterpret_cast<const uint4 *>(gbase + static_cast<size_t>(r0) * 2 * N + 8 * tau);
 #pragma unroll
       for (int c = 0; c < 2; ++c) {
-        const uint4 *g0 = reinterpret_cast<const uint4 *>(gbase + (static_cast<size_t>(r0) * 2 + c) * N + 8 * tau);
-        const uint4 *g1 = reinterpret_cast<const uint4 *>(gbase + (static_cast<size_t>(r0 + 1) * 2 + c) * N + 8 * tau);
-        const uint4 a0 = __ldg(g0), a1 = __ldg(g0 + 1), b0 = __ldg(g1), b1 = __ldg(g1 + 1);
+        const uint4 a0 = __ldg(g + (c * N) / 4), a1 = __ldg(g + (c * N) / 4 + 1);
+        const uint4 b0 = __ldg(g + ((2 + c) * N) / 4), b1 = __ldg(g + ((2 + c) * N) / 4 + 1);
+        if (c == 0) {
+#pragma unroll
+          for (int pp = 0; pp < 2; ++pp)
+#pragma unroll
+            for (int e = 0; e < 8; ++e) x[pp][e] = cond_sub(x[pp][e], 4 * p);  // < 8p -> < 4p
+        }
         const uint32_t ga[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
         const uint32_t gb[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
-          // forward outputs < 8p, brought below 4p; BSK words < p in Montgomery
-          // form, so the pair sum stays below p * 2^32
-          const uint32_t x0 = cond_sub(x[0][e], 4 * p), x1 = cond_sub(x[1][e], 4 * p);
-          const uint64_t prod = static_cast<uint64_t>(x0) * ga[e] + static_cast<uint64_t>(x1) * gb[e];
+          // forward outputs < 4p, BSK words < p in Montgomery form: the pair
+          // sum stays below p * 2^32
+          const uint64_t prod = static_cast<uint64_t>(x[0][e]) * ga[e] + static_cast<uint64_t>(x[1][e]) * gb[e];
           const uint32_t rr = redc(prod, p, p_inv);  // (0, 2p)
           oh[c][e] = (r0 == 0) ? rr : cond_sub(oh[c][e] + rr, 4 * p);
         }
@@ -181,7 +197,7 @@ __global__ void __launch_bounds__((1 << LOGN) / 8) blind_rotate_kernel(const BrA
 #pragma unroll
       for (int q = 0; q < 8; ++q) {
         const uint32_t y = shoup_mul(oh[c][q], crt_c, crt_cs, p);  // [0, 2p)
-        rres[q >> 1][(rank * 2 + c) * Q + tau + (q & 1) * T] = y;
+        dsmem_st_u32(dsmem_map(res_s + ((rank * 2 + c) * Q + tau + (q & 1) * T) * 4u, q >> 1), y);
       }
     cluster.sync();
 
@@ -221,7 +237,7 @@ __global__ void __launch_bounds__((1 << LOGN) / 8) blind_rotate_kernel(const BrA
 
 size_t br_smem_bytes(uint32_t logN, uint32_t level, uint32_t n, bool dig16) {
   const size_t N = size_t(1) << logN, Q = N / 4;
-  const size_t xbuf = (logN <= 11) ? 2 : 1;
+  const size_t xbuf = br_xbuf(static_cast<int>(logN));
   size_t b = N * sizeof(uint2) + 2 * Q * sizeof(uint64_t) + kPrimes * 2 * Q * sizeof(uint32_t) +
              xbuf * (N + N / 8) * sizeof(uint32_t) + 2 * level * Q * (dig16 ? 2 : 4) + (n + 1) * sizeof(uint16_t);
   return (b + 15) & ~size_t(15);
@@ -232,6 +248,8 @@ static cudaError_t launch_br_t(const BrArgs &a, cudaStream_t s) {
   auto kern = blind_rotate_kernel<LOGN, DIG16>;
   const size_t smem = br_smem_bytes(LOGN, a.level, a.n, DIG16);
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(4 * a.batch, 1, 1);

@@ -5,7 +5,7 @@
 #include <stddef.h>
 #include <stdint.h>
 
-#include "../../include/rosetta.h"
+#include "rosetta.h"
 #include "internal.h"
 
 struct rosetta_ctx {

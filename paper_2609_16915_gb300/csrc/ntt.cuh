@@ -77,13 +77,43 @@ __device__ __forceinline__ void ct_bfly(uint32_t &X, uint32_t &Y, uint2 w, uint3
 __host__ __device__ constexpr bool fwd_stage_corrects(int s) { return s >= 3 && ((s - 3) % 2 == 0); }
 
 // Inverse (Gentleman-Sande) butterfly with inverse twiddle -w:
-// X' = X + Y (brought below 4p), Y' = (X - Y)(-w) = (Y - X + 4p) w.
-// Inputs < 4p give X' < 4p and Y' < 2p.
-__device__ __forceinline__ void gs_bfly(uint32_t &X, uint32_t &Y, uint2 w, uint32_t p, uint32_t four_p) {
+// X' = X + Y, Y' = (X - Y)(-w) = (Y - X + 4p) w.  Inputs < 4p give X' < 8p,
+// brought below 4p when CORR, and Y' < 2p.  Both inputs of an inverse
+// butterfly are outputs of the same kind (X' or Y') of the previous stage;
+// when they are Y' outputs (< 2p) their sum is already below 4p and the
+// correction is skipped.
+__device__ __forceinline__ void gs_bfly(uint32_t &X, uint32_t &Y, uint2 w, uint32_t p, uint32_t four_p, bool corr) {
   const uint32_t s = X + Y;
   const uint32_t d = Y - X + four_p;
-  X = cond_sub(s, four_p);
+  X = corr ? cond_sub(s, four_p) : s;  // corr is a constant after unrolling
   Y = shoup_mul(d, w.x, w.y, p);
+}
+
+// Does inverse stage S (inside the pass (S0, H), U = S - S0) need the
+// correction for the butterfly at register position q?  Its inputs come from
+// stage S+1, where the element at q was an X' output iff bit (H - U - 2) of q
+// is 0.  The first stage of every pass (U = H - 1) looks at a bit outside q
+// and always corrects.
+template <int H, int U>
+__host__ __device__ constexpr bool inv_corrects(int q) {
+  return U >= H - 1 ? true : ((q >> (H - U - 2)) & 1) == 0;
+}
+
+// Load CNT (1, 2 or 4) consecutive twiddle pairs starting at an index that is
+// a multiple of CNT: one 8-byte or one/two 16-byte shared-memory loads.
+template <int CNT>
+__device__ __forceinline__ void load_twiddles(const uint2 *__restrict__ tw, uint32_t start, uint2 (&w)[CNT]) {
+  if constexpr (CNT == 1) {
+    w[0] = tw[start];
+  } else {
+    const uint4 *p = reinterpret_cast<const uint4 *>(tw + start);
+#pragma unroll
+    for (int k = 0; k < CNT / 2; ++k) {
+      const uint4 v = p[k];
+      w[2 * k] = make_uint2(v.x, v.y);
+      w[2 * k + 1] = make_uint2(v.z, v.w);
+    }
+  }
 }
 
 template <int LOGN, int NP, int S0, int H, int U>
@@ -95,16 +125,33 @@ __device__ __forceinline__ void fwd_stage(uint32_t (&x)[NP][8], const uint2 *__r
   constexpr int S = S0 + U;
   constexpr int HALF = 1 << (H - 1 - U);
   constexpr bool CORR = fwd_stage_corrects(S);
+  if constexpr (SIG == 1) {
+    // last pass: the thread's groups are consecutive, so are their twiddles
+    constexpr int CNT = NB << U;
+    uint2 w[CNT];
+    load_twiddles<CNT>(tw, (1u << S) + tau * CNT, w);
 #pragma unroll
-  for (int b = 0; b < NB; ++b) {
-    const uint32_t g = (tau * NB + b) / SIG;
+    for (int b = 0; b < NB; ++b)
 #pragma unroll
-    for (int q = 0; q < (1 << H); ++q) {
-      if (q & HALF) continue;
-      const uint2 w = tw[(1u << S) + (g << U) + (q >> (H - U))];
+      for (int q = 0; q < (1 << H); ++q) {
+        if (q & HALF) continue;
 #pragma unroll
-      for (int k = 0; k < NP; ++k)
-        ct_bfly<CORR>(x[k][b * (1 << H) + q], x[k][b * (1 << H) + q + HALF], w, p, two_p, four_p);
+        for (int k = 0; k < NP; ++k)
+          ct_bfly<CORR>(x[k][b * (1 << H) + q], x[k][b * (1 << H) + q + HALF], w[(b << U) + (q >> (H - U))], p, two_p,
+                        four_p);
+      }
+  } else {
+#pragma unroll
+    for (int b = 0; b < NB; ++b) {
+      const uint32_t g = (tau * NB + b) / SIG;
+#pragma unroll
+      for (int q = 0; q < (1 << H); ++q) {
+        if (q & HALF) continue;
+        const uint2 w = tw[(1u << S) + (g << U) + (q >> (H - U))];
+#pragma unroll
+        for (int k = 0; k < NP; ++k)
+          ct_bfly<CORR>(x[k][b * (1 << H) + q], x[k][b * (1 << H) + q + HALF], w, p, two_p, four_p);
+      }
     }
   }
 }
@@ -117,16 +164,35 @@ __device__ __forceinline__ void inv_stage(uint32_t (&x)[NP][8], const uint2 *__r
   constexpr int NB = 8 >> H;
   constexpr int S = S0 + U;
   constexpr int HALF = 1 << (H - 1 - U);
+  if constexpr (SIG == 1) {
+    // last pass: groups G in [tau*CNT, (tau+1)*CNT) use the descending run
+    // W[2^{s+1}-1-G], which starts at 2^{s+1} - (tau+1)*CNT
+    constexpr int CNT = NB << U;
+    uint2 w[CNT];
+    load_twiddles<CNT>(tw, (2u << S) - (tau + 1) * CNT, w);
 #pragma unroll
-  for (int b = 0; b < NB; ++b) {
-    const uint32_t g = (tau * NB + b) / SIG;
+    for (int b = 0; b < NB; ++b)
 #pragma unroll
-    for (int q = 0; q < (1 << H); ++q) {
-      if (q & HALF) continue;
-      const uint32_t G = (g << U) + (q >> (H - U));
-      const uint2 w = tw[(2u << S) - 1u - G];
+      for (int q = 0; q < (1 << H); ++q) {
+        if (q & HALF) continue;
+        const int idx = CNT - 1 - ((b << U) + (q >> (H - U)));
 #pragma unroll
-      for (int k = 0; k < NP; ++k) gs_bfly(x[k][b * (1 << H) + q], x[k][b * (1 << H) + q + HALF], w, p, four_p);
+        for (int k = 0; k < NP; ++k)
+          gs_bfly(x[k][b * (1 << H) + q], x[k][b * (1 << H) + q + HALF], w[idx], p, four_p, inv_corrects<H, U>(q));
+      }
+  } else {
+#pragma unroll
+    for (int b = 0; b < NB; ++b) {
+      const uint32_t g = (tau * NB + b) / SIG;
+#pragma unroll
+      for (int q = 0; q < (1 << H); ++q) {
+        if (q & HALF) continue;
+        const uint32_t G = (g << U) + (q >> (H - U));
+        const uint2 w = tw[(2u << S) - 1u - G];
+#pragma unroll
+        for (int k = 0; k < NP; ++k)
+          gs_bfly(x[k][b * (1 << H) + q], x[k][b * (1 << H) + q + HALF], w, p, four_p, inv_corrects<H, U>(q));
+      }
     }
   }
 }
@@ -147,33 +213,91 @@ __device__ __forceinline__ void inv_pass(uint32_t (&x)[NP][8], const uint2 *tw, 
   inv_stage<LOGN, NP, S0, H, 0>(x, tw, tau, p, four_p);
 }
 
+// A pass whose butterfly groups span at most 256 elements keeps every warp's
+// 32 x 8 values inside one aligned 256-element range, so an exchange between
+// two such passes only needs the warp to synchronise.
+template <int LOGN, int S0>
+__host__ __device__ constexpr bool pass_warp_local() {
+  return (1 << (LOGN - S0)) <= 256;
+}
+
+__host__ __device__ constexpr uint32_t xb_pad_c(uint32_t i) { return i + ((i >> 5) << 2); }
+
+// Padded address of slot e of thread tau in the pass (S0, H), split as a
+// per-thread base plus a compile-time offset: for every pass shape the low
+// five bits of base and offset never carry, so pad(base + off) =
+// pad(base) + pad(off).  Non-last passes have H = 3 and one block per thread
+// (base = g*SPAN + i, offset e*SIG); in the last pass a thread's slots are
+// the 8 consecutive positions 8*tau + e.
+template <int LOGN, int S0, int H>
+__device__ __forceinline__ uint32_t xb_base(uint32_t tau) {
+  constexpr uint32_t N = 1u << LOGN, SIG = N >> (S0 + H), SPAN = N >> S0;
+  if constexpr (SIG == 1) {
+    return xb_pad(8 * tau);
+  } else {
+    static_assert(H == 3, "only the last pass is shorter than three stages");
+    return xb_pad((tau / SIG) * SPAN + tau % SIG);
+  }
+}
+
+template <int LOGN, int S0, int H>
+__host__ __device__ constexpr uint32_t xb_off(int e) {
+  constexpr uint32_t N = 1u << LOGN, SIG = N >> (S0 + H);
+  return xb_pad_c(SIG == 1 ? static_cast<uint32_t>(e) : static_cast<uint32_t>(e) * SIG);
+}
+
+// Store / load one thread's 8 slots of the pass (S0, H).  In the last pass
+// the 8 consecutive words are 16-byte aligned: two vector accesses.
+template <int LOGN, int S0, int H>
+__device__ __forceinline__ void xb_store(uint32_t *buf, const uint32_t (&v)[8], uint32_t tau) {
+  uint32_t *b = buf + xb_base<LOGN, S0, H>(tau);
+  if constexpr (S0 + H == LOGN) {
+    uint4 *p = reinterpret_cast<uint4 *>(b);
+    p[0] = make_uint4(v[0], v[1], v[2], v[3]);
+    p[1] = make_uint4(v[4], v[5], v[6], v[7]);
+  } else {
+#pragma unroll
+    for (int e = 0; e < 8; ++e) b[xb_off<LOGN, S0, H>(e)] = v[e];
+  }
+}
+
+template <int LOGN, int S0, int H>
+__device__ __forceinline__ void xb_load(const uint32_t *buf, uint32_t (&v)[8], uint32_t tau) {
+  const uint32_t *b = buf + xb_base<LOGN, S0, H>(tau);
+  if constexpr (S0 + H == LOGN) {
+    const uint4 *p = reinterpret_cast<const uint4 *>(b);
+    const uint4 a = p[0], c = p[1];
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+    v[4] = c.x; v[5] = c.y; v[6] = c.z; v[7] = c.w;
+  } else {
+#pragma unroll
+    for (int e = 0; e < 8; ++e) v[e] = b[xb_off<LOGN, S0, H>(e)];
+  }
+}
+
 // Move NP register sets from the layout of pass A to that of pass B through
 // the exchange buffer xb (XBUF polynomials of NttShape::XB_WORDS words each).
-// The leading barrier protects xb from readers of the previous exchange.
+// The leading barrier protects xb from readers of the previous exchange; it
+// and the middle one are warp barriers when both passes are warp-local.
 template <int LOGN, int NP, int XBUF, int S0A, int HA, int S0B, int HB>
 __device__ __forceinline__ void exchange(uint32_t (&x)[NP][8], uint32_t *xb, uint32_t tau) {
   constexpr int W = NttShape<LOGN>::XB_WORDS;
+  constexpr bool WARP = pass_warp_local<LOGN, (S0A < S0B ? S0A : S0B)>();
   static_assert(XBUF == 1 || XBUF == NP, "exchange buffer must hold one or all polynomials");
   if constexpr (XBUF == NP) {
-    __syncthreads();
+    if constexpr (WARP) __syncwarp(); else __syncthreads();
 #pragma unroll
-    for (int k = 0; k < NP; ++k)
+    for (int k = 0; k < NP; ++k) xb_store<LOGN, S0A, HA>(xb + k * W, x[k], tau);
+    if constexpr (WARP) __syncwarp(); else __syncthreads();
 #pragma unroll
-      for (int e = 0; e < 8; ++e) xb[k * W + xb_pad(slot_index<LOGN, S0A, HA>(tau, e))] = x[k][e];
-    __syncthreads();
-#pragma unroll
-    for (int k = 0; k < NP; ++k)
-#pragma unroll
-      for (int e = 0; e < 8; ++e) x[k][e] = xb[k * W + xb_pad(slot_index<LOGN, S0B, HB>(tau, e))];
+    for (int k = 0; k < NP; ++k) xb_load<LOGN, S0B, HB>(xb + k * W, x[k], tau);
   } else {
 #pragma unroll
     for (int k = 0; k < NP; ++k) {
-      __syncthreads();
-#pragma unroll
-      for (int e = 0; e < 8; ++e) xb[xb_pad(slot_index<LOGN, S0A, HA>(tau, e))] = x[k][e];
-      __syncthreads();
-#pragma unroll
-      for (int e = 0; e < 8; ++e) x[k][e] = xb[xb_pad(slot_index<LOGN, S0B, HB>(tau, e))];
+      if constexpr (WARP) __syncwarp(); else __syncthreads();
+      xb_store<LOGN, S0A, HA>(xb, x[k], tau);
+      if constexpr (WARP) __syncwarp(); else __syncthreads();
+      xb_load<LOGN, S0B, HB>(xb, x[k], tau);
     }
   }
 }

@@ -7,7 +7,7 @@
 #include <new>
 #include <vector>
 
-#include "../../include/rosetta.h"
+#include "rosetta.h"
 #include "context.h"
 #include "internal.h"
 

@@ -60,6 +60,29 @@ def int_ops_per_pbs(p):
     return per_cmux * p.n, ks
 
 
+TRAFFIC_SUMMARY = os.path.join(ROOT, "profiles", "blind_rotate_standard_b4096_dram.txt")
+
+
+def measured_traffic(p, batch):
+    """DRAM bytes (read + write) of one blind-rotation launch from the
+    committed ncu summary, or None when the summary is for another workload
+    or the kernel sources changed since it was captured."""
+    import hashlib
+    try:
+        kv = dict(line.strip().split("=", 1) for line in open(TRAFFIC_SUMMARY)
+                  if "=" in line and not line.startswith("#"))
+    except OSError:
+        return None
+    if kv.get("config") != p.name or int(kv.get("batch", -1)) != batch:
+        return None
+    h = hashlib.sha256()
+    for f in kv["sources"].split(","):
+        h.update(open(os.path.join(ROOT, "paper_2609_16915_gb300", "csrc", f), "rb").read())
+    if h.hexdigest() != kv.get("sources_sha256"):
+        return None
+    return int(kv["dram_bytes_read"]) + int(kv["dram_bytes_write"])
+
+
 def peaks():
     try:
         return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
@@ -197,6 +220,7 @@ def main():
     torch.cuda.set_device(dev)
 
     import paper_2609_16915_gb300 as R
+    from paper_2609_16915_gb300 import multi
     R.load()
 
     def d(a):
@@ -241,10 +265,7 @@ def main():
     ctx.sync_status(stream)
     step_ms = [a.elapsed_time(b) for a, b in ev]
     total_ms = sum(step_ms)
-    t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
-    if dist:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    total_ms = float(t.item())
+    total_ms = multi.max_over_ranks(total_ms, dist, dev)
     value = world * batch * args.steps / (total_ms / 1e3)
 
     # dominant kernel (blind rotation) alone, same launch, events on its stream
@@ -274,10 +295,7 @@ def main():
     for _ in range(e2e_steps):
         ctx.pbs_batch(h_in, h_lut, h_out, stream)   # copies in, PBS, copies out, synchronises
     e2e_s = (time.perf_counter() - t0) / e2e_steps
-    e2e_t = torch.tensor([e2e_s], dtype=torch.float64, device=dev)
-    if dist:
-        dist.all_reduce(e2e_t, op=dist.ReduceOp.MAX)
-    e2e_value = world * batch / float(e2e_t.item())
+    e2e_value = world * batch / multi.max_over_ranks(e2e_s, dist, dev)
 
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
     pk = peaks()
@@ -298,7 +316,7 @@ def main():
         "config": {"workload": describe(p, batch), "batch": batch, "parallelism": f"dp{world}" if world > 1 else "none",
                    "l2": "flushed between steps (256 MB write)", "keys": "uniform words, resident"},
         "roofline": {"bound": "alu", "kernel": "blind_rotate_kernel", "achieved": achieved, "peak": alu_peak,
-                     "unit": "Tops/s (int32)", "frac": achieved / alu_peak, "traffic": None,
+                     "unit": "Tops/s (int32)", "frac": achieved / alu_peak, "traffic": measured_traffic(p, batch),
                      "peak_basis": f"{sms} SMs x 128 int32 lanes x {sm_max:.0f} MHz (sm_max_mhz of MEASURED_PEAKS.json)",
                      "kernel_ms": br_ms, "keyswitch_ms": ks_ms,
                      "pbs_roof": pbs_roof, "pbs_frac_of_roof": value / world / pbs_roof},

@@ -13,15 +13,18 @@
 namespace rosetta {
 
 namespace {
-constexpr int KS_BM = 64, KS_BN = 64, KS_TM = 4, KS_TN = 4, KS_KI = 8;
+// 64 ciphertexts x 64 output words per CTA; 128 threads, each 8 ciphertexts x
+// 4 consecutive output words; KS_KI input coefficients (KS_KI * l rows of the
+// KSK) per shared-memory tile.
+constexpr int KS_BM = 64, KS_BN = 64, KS_TM = 8, KS_TN = 4, KS_KI = 8;
 constexpr int KS_THREADS = (KS_BM / KS_TM) * (KS_BN / KS_TN);
 }  // namespace
 
 __global__ void __launch_bounds__(KS_THREADS) keyswitch_kernel(const KsArgs a) {
   extern __shared__ __align__(16) unsigned char smem[];
   const uint32_t level = a.level;
-  uint64_t *ks = reinterpret_cast<uint64_t *>(smem);                  // [KI*level][BN]
-  uint32_t *dg = reinterpret_cast<uint32_t *>(ks + KS_KI * level * KS_BN);  // [KI*level][BM]
+  uint64_t *ks = reinterpret_cast<uint64_t *>(smem);                          // [KI*level][BN]
+  uint32_t *dg = reinterpret_cast<uint32_t *>(ks + KS_KI * level * KS_BN);    // [KI*level][BM]
   const uint32_t tid = threadIdx.x;
   const uint32_t tx = tid % (KS_BN / KS_TN), ty = tid / (KS_BN / KS_TN);
   const uint32_t b0 = blockIdx.y * KS_BM, o0 = blockIdx.x * KS_BN;
@@ -43,15 +46,15 @@ __global__ void __launch_bounds__(KS_THREADS) keyswitch_kernel(const KsArgs a) {
   for (uint32_t i0 = 0; i0 < a.kN; i0 += KS_KI) {
     __syncthreads();
     for (uint32_t idx = tid; idx < KS_BM * KS_KI; idx += KS_THREADS) {
-      const uint32_t m = idx / KS_KI, ii = idx % KS_KI;
+      const uint32_t ii = idx % KS_KI, m = idx / KS_KI;  // consecutive words of one ciphertext
       const uint32_t b = b0 + m, i = i0 + ii;
       const uint64_t v = (b < a.batch && i < a.kN) ? a.big[static_cast<size_t>(b) * stride_in + i] : 0;
       uint64_t cv = bits >= 64 ? v : (v + (1ull << (63 - bits))) >> (64 - bits);
       for (int l = static_cast<int>(level) - 1; l >= 0; --l) {
-        uint64_t d = cv & Bmask;
+        const uint64_t d = cv & Bmask;
         cv >>= a.base_log;
         if (d >= Bhalf) cv += 1;
-        // d - B/2 mod B re-centres the balanced digit: shifted digit = (d + B/2) mod B
+        // the balanced digit d or d - B, shifted by B/2 into [0, B)
         dg[(ii * level + l) * KS_BM + m] = static_cast<uint32_t>((d + Bhalf) & Bmask);
       }
     }
@@ -62,28 +65,29 @@ __global__ void __launch_bounds__(KS_THREADS) keyswitch_kernel(const KsArgs a) {
     }
     __syncthreads();
     for (uint32_t kr = 0; kr < krows; ++kr) {
-      uint32_t d[KS_TM];
-      uint64_t g[KS_TN];
-#pragma unroll
-      for (int m = 0; m < KS_TM; ++m) d[m] = dg[kr * KS_BM + ty + m * (KS_BM / KS_TM)];
-#pragma unroll
-      for (int t = 0; t < KS_TN; ++t) g[t] = ks[kr * KS_BN + tx + t * (KS_BN / KS_TN)];
+      const uint4 d0 = *reinterpret_cast<const uint4 *>(dg + kr * KS_BM + ty * KS_TM);
+      const uint4 d1 = *reinterpret_cast<const uint4 *>(dg + kr * KS_BM + ty * KS_TM + 4);
+      const uint4 g01 = *reinterpret_cast<const uint4 *>(ks + kr * KS_BN + tx * KS_TN);
+      const uint4 g23 = *reinterpret_cast<const uint4 *>(ks + kr * KS_BN + tx * KS_TN + 2);
+      const uint32_t d[KS_TM] = {d0.x, d0.y, d0.z, d0.w, d1.x, d1.y, d1.z, d1.w};
+      const uint32_t glo[KS_TN] = {g01.x, g01.z, g23.x, g23.z};
+      const uint32_t ghi[KS_TN] = {g01.y, g01.w, g23.y, g23.w};
 #pragma unroll
       for (int m = 0; m < KS_TM; ++m)
 #pragma unroll
         for (int t = 0; t < KS_TN; ++t) {
-          lo[m][t] += static_cast<uint64_t>(d[m]) * static_cast<uint32_t>(g[t]);
-          hi[m][t] += d[m] * static_cast<uint32_t>(g[t] >> 32);
+          lo[m][t] += static_cast<uint64_t>(d[m]) * glo[t];
+          hi[m][t] += d[m] * ghi[t];
         }
     }
   }
 #pragma unroll
   for (int m = 0; m < KS_TM; ++m) {
-    const uint32_t b = b0 + ty + m * (KS_BM / KS_TM);
+    const uint32_t b = b0 + ty * KS_TM + m;
     if (b >= a.batch) continue;
 #pragma unroll
     for (int t = 0; t < KS_TN; ++t) {
-      const uint32_t o = o0 + tx + t * (KS_BN / KS_TN);
+      const uint32_t o = o0 + tx * KS_TN + t;
       if (o >= n1) continue;
       const uint64_t sum = lo[m][t] + (static_cast<uint64_t>(hi[m][t]) << 32);
       const uint64_t body = (o == a.n) ? a.big[static_cast<size_t>(b) * stride_in + a.kN] : 0;

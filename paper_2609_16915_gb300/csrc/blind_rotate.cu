@@ -43,11 +43,20 @@ namespace cg = cooperative_groups;
 // plentiful; larger rings share one buffer to keep more CTAs resident.
 __host__ __device__ constexpr int br_xbuf(int logN) { return logN <= 10 ? 2 : 1; }
 
+// Values per thread in the transforms.  16 halves the CTA-wide exchanges but
+// also the warps per SM; measured on GB300 it is slower at every ring size
+// (N = 2048: 309 vs 276 ms, 4096: 822 vs 782 ms, 8192: 14.0 vs 12.8 s for the
+// full batches), so 8 is used throughout.
+__host__ __device__ constexpr int br_e(int) { return 8; }
+
 template <int LOGN>
 struct BrShape {
   static constexpr int N = 1 << LOGN;
-  static constexpr int T = N / 8;
+  static constexpr int E = br_e(LOGN);
+  static constexpr int T = N / E;                      // threads per CTA
   static constexpr int Q = N / 4;                      // coefficients owned per CTA
+  static constexpr int ITEMS = 2 * Q / T;              // owned (component, coefficient) pairs per thread
+  static constexpr int QE = E / 4;                     // first-pass slots per owner quarter
   static constexpr int XBUF = br_xbuf(LOGN);            // exchange buffers (polys)
   // resident CTAs per SM the register allocation must allow (shared memory
   // allows the same: 4 x 55 KB at N = 2048, 2 x 108 KB at 4096)
@@ -55,11 +64,12 @@ struct BrShape {
 };
 
 template <int LOGN, bool DIG16>
-__global__ void __launch_bounds__((1 << LOGN) / 8, BrShape<LOGN>::MIN_CTAS) blind_rotate_kernel(const BrArgs a) {
-  using S = NttShape<LOGN>;
+__global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) blind_rotate_kernel(const BrArgs a) {
   using B = BrShape<LOGN>;
+  using S = NttShape<LOGN, B::E>;
   using DigT = typename std::conditional<DIG16, int16_t, int32_t>::type;
   constexpr uint32_t N = B::N, T = B::T, Q = B::Q;
+  constexpr int E = B::E, ITEMS = B::ITEMS, QE = B::QE;
   constexpr uint32_t TWO_N = 2 * N;
 
   cg::cluster_group cluster = cg::this_cluster();
@@ -91,7 +101,7 @@ __global__ void __launch_bounds__((1 << LOGN) / 8, BrShape<LOGN>::MIN_CTAS) blin
     const uint32_t btil = atil[a.n];
     const uint32_t box = N >> a.msg_bits, h = box >> 1;
 #pragma unroll
-    for (int m = 0; m < 4; ++m) {
+    for (int m = 0; m < ITEMS; ++m) {
       const uint32_t item = tau + m * T;
       const uint32_t c = item / Q, jl = item % Q, j = rank * Q + jl;
       if (c == 0) {
@@ -122,18 +132,18 @@ __global__ void __launch_bounds__((1 << LOGN) / 8, BrShape<LOGN>::MIN_CTAS) blin
     if (at == 0) continue;  // X^0 ACC - ACC = 0: the step adds nothing
 
     // ---- phase 1: rotated difference and gadget digits of the owned quarter ----
-    // (X^a P)[j] = +-P[(j - a) mod 2N]; the four remote words are requested
+    // (X^a P)[j] = +-P[(j - a) mod 2N]; all remote words are requested
     // before any is used so their latencies overlap
-    uint64_t v[4];
+    uint64_t v[ITEMS];
 #pragma unroll
-    for (int m = 0; m < 4; ++m) {
+    for (int m = 0; m < ITEMS; ++m) {
       const uint32_t item = tau + m * T;
       const uint32_t c = item / Q, jl = item % Q, j = rank * Q + jl;
       const uint32_t e = (j + TWO_N - at) & (N - 1);
       v[m] = dsmem_ld_u64(dsmem_map(acc_s + (c * Q + (e % Q)) * 8u, e / Q));
     }
 #pragma unroll
-    for (int m = 0; m < 4; ++m) {
+    for (int m = 0; m < ITEMS; ++m) {
       const uint32_t item = tau + m * T;
       const uint32_t c = item / Q, jl = item % Q, j = rank * Q + jl;
       const bool neg = ((j + TWO_N - at) & (TWO_N - 1)) >= N;
@@ -153,36 +163,41 @@ __global__ void __launch_bounds__((1 << LOGN) / 8, BrShape<LOGN>::MIN_CTAS) blin
     cluster.sync();
 
     // ---- phase 2: transforms and pointwise products for prime `rank` ----
-    uint32_t oh[2][8];
+    uint32_t oh[2][E];
     const uint32_t *gbase = a.bsk + (static_cast<size_t>(i) * kPrimes + rank) * (static_cast<size_t>(L2) * 2 * N);
     for (uint32_t r0 = 0; r0 < L2; r0 += 2) {
-      uint32_t x[2][8];
+      // first-pass slot q of thread tau is coefficient tau + q N/E, owned by
+      // CTA q / QE at local index tau + (q % QE) T
+      uint32_t x[2][E];
 #pragma unroll
       for (int pp = 0; pp < 2; ++pp)
 #pragma unroll
-        for (int q = 0; q < 8; ++q) {
-          const uint32_t ad = dsmem_map(dig_s + ((r0 + pp) * Q + tau + (q & 1) * T) * sizeof(DigT), q >> 1);
+        for (int q = 0; q < E; ++q) {
+          const uint32_t ad = dsmem_map(dig_s + ((r0 + pp) * Q + tau + (q % QE) * T) * sizeof(DigT), q / QE);
           const int32_t d = DIG16 ? dsmem_ld_s16(ad) : dsmem_ld_s32(ad);
           x[pp][q] = static_cast<uint32_t>(d + static_cast<int32_t>(p));  // in (0, 2p)
         }
-      ntt_forward<LOGN, 2, B::XBUF>(x, tw, xb, tau, p);
-      // BSK_i words of this prime for rows r0, r0+1, 8 per thread and
+      ntt_forward<LOGN, E, 2, B::XBUF>(x, tw, xb, tau, p);
+      // BSK_i words of this prime for rows r0, r0+1, E per thread and
       // component, contiguous across the CTA (16-byte loads)
-      const uint4 *g = reinterpret_cast<const uint4 *>(gbase + static_cast<size_t>(r0) * 2 * N + 8 * tau);
+      const uint4 *g = reinterpret_cast<const uint4 *>(gbase + static_cast<size_t>(r0) * 2 * N + E * tau);
 #pragma unroll
       for (int c = 0; c < 2; ++c) {
-        const uint4 a0 = __ldg(g + (c * N) / 4), a1 = __ldg(g + (c * N) / 4 + 1);
-        const uint4 b0 = __ldg(g + ((2 + c) * N) / 4), b1 = __ldg(g + ((2 + c) * N) / 4 + 1);
+        uint32_t ga[E], gb[E];
+#pragma unroll
+        for (int k = 0; k < E / 4; ++k) {
+          const uint4 va = __ldg(g + (c * N) / 4 + k), vb = __ldg(g + ((2 + c) * N) / 4 + k);
+          ga[4 * k] = va.x; ga[4 * k + 1] = va.y; ga[4 * k + 2] = va.z; ga[4 * k + 3] = va.w;
+          gb[4 * k] = vb.x; gb[4 * k + 1] = vb.y; gb[4 * k + 2] = vb.z; gb[4 * k + 3] = vb.w;
+        }
         if (c == 0) {
 #pragma unroll
           for (int pp = 0; pp < 2; ++pp)
 #pragma unroll
-            for (int e = 0; e < 8; ++e) x[pp][e] = cond_sub(x[pp][e], 4 * p);  // < 8p -> < 4p
+            for (int e = 0; e < E; ++e) x[pp][e] = cond_sub(x[pp][e], 4 * p);  // < 8p -> < 4p
         }
-        const uint32_t ga[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
-        const uint32_t gb[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
+        for (int e = 0; e < E; ++e) {
           // forward outputs < 4p, BSK words < p in Montgomery form: the pair
           // sum stays below p * 2^32
           const uint64_t prod = static_cast<uint64_t>(x[0][e]) * ga[e] + static_cast<uint64_t>(x[1][e]) * gb[e];
@@ -191,19 +206,19 @@ __global__ void __launch_bounds__((1 << LOGN) / 8, BrShape<LOGN>::MIN_CTAS) blin
         }
       }
     }
-    ntt_inverse<LOGN, 2, B::XBUF>(oh, tw, xb, tau, p);
+    ntt_inverse<LOGN, E, 2, B::XBUF>(oh, tw, xb, tau, p);
 #pragma unroll
     for (int c = 0; c < 2; ++c)
 #pragma unroll
-      for (int q = 0; q < 8; ++q) {
+      for (int q = 0; q < E; ++q) {
         const uint32_t y = shoup_mul(oh[c][q], crt_c, crt_cs, p);  // [0, 2p)
-        dsmem_st_u32(dsmem_map(res_s + ((rank * 2 + c) * Q + tau + (q & 1) * T) * 4u, q >> 1), y);
+        dsmem_st_u32(dsmem_map(res_s + ((rank * 2 + c) * Q + tau + (q % QE) * T) * 4u, q / QE), y);
       }
     cluster.sync();
 
     // ---- phase 3: explicit CRT of the owned quarter, accumulate ----
 #pragma unroll
-    for (int m = 0; m < 4; ++m) {
+    for (int m = 0; m < ITEMS; ++m) {
       const uint32_t item = tau + m * T;
       const uint32_t c = item / Q, jl = item % Q;
       uint64_t s = 0;
@@ -223,7 +238,7 @@ __global__ void __launch_bounds__((1 << LOGN) / 8, BrShape<LOGN>::MIN_CTAS) blin
   // ---- sample extraction of the constant coefficient ----
   uint64_t *out = a.lwe_big_out + static_cast<size_t>(ct) * (N + 1);
 #pragma unroll
-  for (int m = 0; m < 4; ++m) {
+  for (int m = 0; m < ITEMS; ++m) {
     const uint32_t item = tau + m * T;
     const uint32_t c = item / Q, jl = item % Q, j = rank * Q + jl;
     if (c == 0) {
@@ -253,7 +268,7 @@ static cudaError_t launch_br_t(const BrArgs &a, cudaStream_t s) {
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(4 * a.batch, 1, 1);
-  cfg.blockDim = dim3((1 << LOGN) / 8, 1, 1);
+  cfg.blockDim = dim3(BrShape<LOGN>::T, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];

@@ -17,7 +17,7 @@ template <int LOGN>
 __global__ void __launch_bounds__((1 << LOGN) / 8)
     bsk_transform_kernel(const uint64_t *__restrict__ raw, uint32_t *__restrict__ out, const uint2 *__restrict__ tw_all,
                          const CrtConsts cc, uint32_t rows) {
-  using S = NttShape<LOGN>;
+  using S = NttShape<LOGN, 8>;
   constexpr uint32_t N = S::N, T = S::T;
   extern __shared__ __align__(16) unsigned char smem[];
   uint2 *tw = reinterpret_cast<uint2 *>(smem);
@@ -40,7 +40,7 @@ __global__ void __launch_bounds__((1 << LOGN) / 8)
     x[0][e] = (neg && r) ? p - r : r;
   }
   __syncthreads();
-  ntt_forward<LOGN, 1, 1>(x, tw, xb, tau, p);
+  ntt_forward<LOGN, 8, 1, 1>(x, tw, xb, tau, p);
 
   const uint32_t c = poly % 2;
   const uint32_t r = (poly / 2) % rows;
@@ -57,7 +57,7 @@ __global__ void __launch_bounds__((1 << LOGN) / 8)
 template <int LOGN>
 static cudaError_t launch_bsk_t(const uint64_t *raw, uint32_t *out, const uint2 *tw, const CrtConsts &cc, uint32_t n,
                                 uint32_t level, cudaStream_t s) {
-  using S = NttShape<LOGN>;
+  using S = NttShape<LOGN, 8>;
   const size_t smem = S::N * sizeof(uint2) + S::XB_WORDS * sizeof(uint32_t);
   auto kern = bsk_transform_kernel<LOGN>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));

@@ -1,5 +1,6 @@
 // Negacyclic number-theoretic transforms of size N = 2^LOGN over one prime,
-// distributed over N/8 threads that each hold 8 residues in registers.
+// distributed over N/E threads that each hold E = 8 or 16 residues in
+// registers.
 //
 // Forward: Cooley-Tukey butterflies with the negacyclic twist merged into the
 // twiddles (W[m] = psi^{bitrev(m)}, psi a primitive 2N-th root of unity);
@@ -9,13 +10,13 @@
 // stage s, group g is psi^{-bitrev(2^s+g)} = -W[2^{s+1}-1-g], so one table
 // serves both directions.
 //
-// The log2(N) stages are grouped into radix-8 passes of three stages (the
-// last pass takes the remaining one to three).  Within a pass each thread
-// owns whole butterfly blocks and keeps them in registers; between passes the
-// values are exchanged through a shared-memory buffer.  After the last
-// forward pass thread t holds bit-reversed positions 8t .. 8t+7, which is
-// exactly what the first inverse pass needs, so a pointwise product between
-// the two transforms needs no exchange.
+// The log2(N) stages are grouped into passes of log2(E) stages (the last pass
+// takes what remains).  Within a pass each thread owns whole butterfly blocks
+// and keeps them in registers; between passes the values are exchanged
+// through a shared-memory buffer.  After the last forward pass thread t holds
+// bit-reversed positions E t .. E t + E-1, which is exactly what the first
+// inverse pass needs, so a pointwise product between the two transforms
+// needs no exchange.
 //
 // Lazy ranges: forward input < 2p, output < 8p; inverse input < 4p, output
 // < 4p.  See the butterflies for the per-stage invariants.
@@ -26,32 +27,37 @@
 
 namespace rosetta {
 
-template <int LOGN>
+__host__ __device__ constexpr int ilog2(int x) { return x <= 1 ? 0 : 1 + ilog2(x >> 1); }
+
+template <int LOGN, int E = 8>
 struct NttShape {
+  static_assert(E == 8 || E == 16, "8 or 16 values per thread");
   static constexpr int N = 1 << LOGN;
-  static constexpr int T = N / 8;                    // threads per transform
-  static constexpr int NPASS = (LOGN + 2) / 3;
-  static constexpr int LAST_H = LOGN - 3 * (NPASS - 1);
+  static constexpr int T = N / E;                    // threads per transform
+  static constexpr int RAD = ilog2(E);               // stages per full pass
+  static constexpr int NPASS = (LOGN + RAD - 1) / RAD;
+  static constexpr int LAST_H = LOGN - RAD * (NPASS - 1);
   static constexpr int XB_WORDS = N + N / 8;         // padded exchange buffer
   template <int PASS>
-  __host__ __device__ static constexpr int h() { return PASS == NPASS - 1 ? LAST_H : 3; }
+  __host__ __device__ static constexpr int h() { return PASS == NPASS - 1 ? LAST_H : RAD; }
 };
 
-// Exchange-buffer address: 4 pad words after every 32 keeps every pass's
-// scalar accesses free of bank conflicts except the last pass, whose
-// contiguous 8-word groups are then read and written as two 16-byte vectors.
+// Exchange-buffer address: 4 pad words after every 32 keeps the scalar
+// accesses of the passes (nearly) free of bank conflicts; the last pass, whose
+// E consecutive words per thread stay 16-byte aligned, uses vector accesses.
 __device__ __forceinline__ uint32_t xb_pad(uint32_t i) { return i + ((i >> 5) << 2); }
+__host__ __device__ constexpr uint32_t xb_pad_c(uint32_t i) { return i + ((i >> 5) << 2); }
 
 // Position (in the stage-ordered data array) of register slot e of thread
 // tau during the pass that starts at stage S0 and spans H stages.  Blocks of
 // 2^H elements have stride SIG = N >> (S0+H) and live in the stage-S0 group
-// g of span N >> S0; a thread owns 8 >> H consecutive blocks.
-template <int LOGN, int S0, int H>
+// g of span N >> S0; a thread owns E >> H consecutive blocks.
+template <int LOGN, int E, int S0, int H>
 __device__ __forceinline__ uint32_t slot_index(uint32_t tau, int e) {
   constexpr uint32_t N = 1u << LOGN;
   constexpr uint32_t SIG = N >> (S0 + H);
   constexpr uint32_t SPAN = N >> S0;
-  constexpr int NB = 8 >> H;
+  constexpr int NB = E >> H;
   const int b = e >> H;
   const int q = e & ((1 << H) - 1);
   const uint32_t beta = tau * NB + b;
@@ -78,7 +84,7 @@ __host__ __device__ constexpr bool fwd_stage_corrects(int s) { return s >= 3 && 
 
 // Inverse (Gentleman-Sande) butterfly with inverse twiddle -w:
 // X' = X + Y, Y' = (X - Y)(-w) = (Y - X + 4p) w.  Inputs < 4p give X' < 8p,
-// brought below 4p when CORR, and Y' < 2p.  Both inputs of an inverse
+// brought below 4p when corr, and Y' < 2p.  Both inputs of an inverse
 // butterfly are outputs of the same kind (X' or Y') of the previous stage;
 // when they are Y' outputs (< 2p) their sum is already below 4p and the
 // correction is skipped.
@@ -99,8 +105,8 @@ __host__ __device__ constexpr bool inv_corrects(int q) {
   return U >= H - 1 ? true : ((q >> (H - U - 2)) & 1) == 0;
 }
 
-// Load CNT (1, 2 or 4) consecutive twiddle pairs starting at an index that is
-// a multiple of CNT: one 8-byte or one/two 16-byte shared-memory loads.
+// Load CNT (a power of two) consecutive twiddle pairs starting at an index
+// that is a multiple of CNT: one 8-byte or CNT/2 16-byte shared loads.
 template <int CNT>
 __device__ __forceinline__ void load_twiddles(const uint2 *__restrict__ tw, uint32_t start, uint2 (&w)[CNT]) {
   if constexpr (CNT == 1) {
@@ -116,12 +122,12 @@ __device__ __forceinline__ void load_twiddles(const uint2 *__restrict__ tw, uint
   }
 }
 
-template <int LOGN, int NP, int S0, int H, int U>
-__device__ __forceinline__ void fwd_stage(uint32_t (&x)[NP][8], const uint2 *__restrict__ tw, uint32_t tau,
+template <int LOGN, int E, int NP, int S0, int H, int U>
+__device__ __forceinline__ void fwd_stage(uint32_t (&x)[NP][E], const uint2 *__restrict__ tw, uint32_t tau,
                                           uint32_t p, uint32_t two_p, uint32_t four_p) {
   constexpr uint32_t N = 1u << LOGN;
   constexpr uint32_t SIG = N >> (S0 + H);
-  constexpr int NB = 8 >> H;
+  constexpr int NB = E >> H;
   constexpr int S = S0 + U;
   constexpr int HALF = 1 << (H - 1 - U);
   constexpr bool CORR = fwd_stage_corrects(S);
@@ -156,12 +162,12 @@ __device__ __forceinline__ void fwd_stage(uint32_t (&x)[NP][8], const uint2 *__r
   }
 }
 
-template <int LOGN, int NP, int S0, int H, int U>
-__device__ __forceinline__ void inv_stage(uint32_t (&x)[NP][8], const uint2 *__restrict__ tw, uint32_t tau,
+template <int LOGN, int E, int NP, int S0, int H, int U>
+__device__ __forceinline__ void inv_stage(uint32_t (&x)[NP][E], const uint2 *__restrict__ tw, uint32_t tau,
                                           uint32_t p, uint32_t four_p) {
   constexpr uint32_t N = 1u << LOGN;
   constexpr uint32_t SIG = N >> (S0 + H);
-  constexpr int NB = 8 >> H;
+  constexpr int NB = E >> H;
   constexpr int S = S0 + U;
   constexpr int HALF = 1 << (H - 1 - U);
   if constexpr (SIG == 1) {
@@ -197,81 +203,82 @@ __device__ __forceinline__ void inv_stage(uint32_t (&x)[NP][8], const uint2 *__r
   }
 }
 
-template <int LOGN, int NP, int S0, int H>
-__device__ __forceinline__ void fwd_pass(uint32_t (&x)[NP][8], const uint2 *tw, uint32_t tau, uint32_t p,
+template <int LOGN, int E, int NP, int S0, int H, int U = 0>
+__device__ __forceinline__ void fwd_pass(uint32_t (&x)[NP][E], const uint2 *tw, uint32_t tau, uint32_t p,
                                          uint32_t two_p, uint32_t four_p) {
-  fwd_stage<LOGN, NP, S0, H, 0>(x, tw, tau, p, two_p, four_p);
-  if constexpr (H > 1) fwd_stage<LOGN, NP, S0, H, 1>(x, tw, tau, p, two_p, four_p);
-  if constexpr (H > 2) fwd_stage<LOGN, NP, S0, H, 2>(x, tw, tau, p, two_p, four_p);
+  fwd_stage<LOGN, E, NP, S0, H, U>(x, tw, tau, p, two_p, four_p);
+  if constexpr (U + 1 < H) fwd_pass<LOGN, E, NP, S0, H, U + 1>(x, tw, tau, p, two_p, four_p);
 }
 
-template <int LOGN, int NP, int S0, int H>
-__device__ __forceinline__ void inv_pass(uint32_t (&x)[NP][8], const uint2 *tw, uint32_t tau, uint32_t p,
+template <int LOGN, int E, int NP, int S0, int H, int U = H - 1>
+__device__ __forceinline__ void inv_pass(uint32_t (&x)[NP][E], const uint2 *tw, uint32_t tau, uint32_t p,
                                          uint32_t four_p) {
-  if constexpr (H > 2) inv_stage<LOGN, NP, S0, H, 2>(x, tw, tau, p, four_p);
-  if constexpr (H > 1) inv_stage<LOGN, NP, S0, H, 1>(x, tw, tau, p, four_p);
-  inv_stage<LOGN, NP, S0, H, 0>(x, tw, tau, p, four_p);
+  inv_stage<LOGN, E, NP, S0, H, U>(x, tw, tau, p, four_p);
+  if constexpr (U > 0) inv_pass<LOGN, E, NP, S0, H, U - 1>(x, tw, tau, p, four_p);
 }
 
-// A pass whose butterfly groups span at most 256 elements keeps every warp's
-// 32 x 8 values inside one aligned 256-element range, so an exchange between
-// two such passes only needs the warp to synchronise.
-template <int LOGN, int S0>
+// A pass whose butterfly groups span at most 32 E elements keeps every
+// warp's 32 x E values inside one aligned range of that size, so an exchange
+// between two such passes only needs the warp to synchronise.
+template <int LOGN, int E, int S0>
 __host__ __device__ constexpr bool pass_warp_local() {
-  return (1 << (LOGN - S0)) <= 256;
+  return (1 << (LOGN - S0)) <= 32 * E;
 }
-
-__host__ __device__ constexpr uint32_t xb_pad_c(uint32_t i) { return i + ((i >> 5) << 2); }
 
 // Padded address of slot e of thread tau in the pass (S0, H), split as a
 // per-thread base plus a compile-time offset: for every pass shape the low
 // five bits of base and offset never carry, so pad(base + off) =
-// pad(base) + pad(off).  Non-last passes have H = 3 and one block per thread
+// pad(base) + pad(off).  Non-last passes have one block per thread
 // (base = g*SPAN + i, offset e*SIG); in the last pass a thread's slots are
-// the 8 consecutive positions 8*tau + e.
-template <int LOGN, int S0, int H>
+// the E consecutive positions E*tau + e.
+template <int LOGN, int E, int S0, int H>
 __device__ __forceinline__ uint32_t xb_base(uint32_t tau) {
   constexpr uint32_t N = 1u << LOGN, SIG = N >> (S0 + H), SPAN = N >> S0;
   if constexpr (SIG == 1) {
-    return xb_pad(8 * tau);
+    return xb_pad(E * tau);
   } else {
-    static_assert(H == 3, "only the last pass is shorter than three stages");
+    static_assert((1 << H) == E, "only the last pass is shorter than a full pass");
     return xb_pad((tau / SIG) * SPAN + tau % SIG);
   }
 }
 
-template <int LOGN, int S0, int H>
+template <int LOGN, int E, int S0, int H>
 __host__ __device__ constexpr uint32_t xb_off(int e) {
   constexpr uint32_t N = 1u << LOGN, SIG = N >> (S0 + H);
   return xb_pad_c(SIG == 1 ? static_cast<uint32_t>(e) : static_cast<uint32_t>(e) * SIG);
 }
 
-// Store / load one thread's 8 slots of the pass (S0, H).  In the last pass
-// the 8 consecutive words are 16-byte aligned: two vector accesses.
-template <int LOGN, int S0, int H>
-__device__ __forceinline__ void xb_store(uint32_t *buf, const uint32_t (&v)[8], uint32_t tau) {
-  uint32_t *b = buf + xb_base<LOGN, S0, H>(tau);
+// Store / load one thread's E slots of the pass (S0, H).  In the last pass the
+// E consecutive words are 16-byte aligned: E/4 vector accesses.
+template <int LOGN, int E, int S0, int H>
+__device__ __forceinline__ void xb_store(uint32_t *buf, const uint32_t (&v)[E], uint32_t tau) {
+  uint32_t *b = buf + xb_base<LOGN, E, S0, H>(tau);
   if constexpr (S0 + H == LOGN) {
     uint4 *p = reinterpret_cast<uint4 *>(b);
-    p[0] = make_uint4(v[0], v[1], v[2], v[3]);
-    p[1] = make_uint4(v[4], v[5], v[6], v[7]);
+#pragma unroll
+    for (int k = 0; k < E / 4; ++k) p[k] = make_uint4(v[4 * k], v[4 * k + 1], v[4 * k + 2], v[4 * k + 3]);
   } else {
 #pragma unroll
-    for (int e = 0; e < 8; ++e) b[xb_off<LOGN, S0, H>(e)] = v[e];
+    for (int e = 0; e < E; ++e) b[xb_off<LOGN, E, S0, H>(e)] = v[e];
   }
 }
 
-template <int LOGN, int S0, int H>
-__device__ __forceinline__ void xb_load(const uint32_t *buf, uint32_t (&v)[8], uint32_t tau) {
-  const uint32_t *b = buf + xb_base<LOGN, S0, H>(tau);
+template <int LOGN, int E, int S0, int H>
+__device__ __forceinline__ void xb_load(const uint32_t *buf, uint32_t (&v)[E], uint32_t tau) {
+  const uint32_t *b = buf + xb_base<LOGN, E, S0, H>(tau);
   if constexpr (S0 + H == LOGN) {
     const uint4 *p = reinterpret_cast<const uint4 *>(b);
-    const uint4 a = p[0], c = p[1];
-    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
-    v[4] = c.x; v[5] = c.y; v[6] = c.z; v[7] = c.w;
+#pragma unroll
+    for (int k = 0; k < E / 4; ++k) {
+      const uint4 a = p[k];
+      v[4 * k] = a.x;
+      v[4 * k + 1] = a.y;
+      v[4 * k + 2] = a.z;
+      v[4 * k + 3] = a.w;
+    }
   } else {
 #pragma unroll
-    for (int e = 0; e < 8; ++e) v[e] = b[xb_off<LOGN, S0, H>(e)];
+    for (int e = 0; e < E; ++e) v[e] = b[xb_off<LOGN, E, S0, H>(e)];
   }
 }
 
@@ -279,56 +286,56 @@ __device__ __forceinline__ void xb_load(const uint32_t *buf, uint32_t (&v)[8], u
 // the exchange buffer xb (XBUF polynomials of NttShape::XB_WORDS words each).
 // The leading barrier protects xb from readers of the previous exchange; it
 // and the middle one are warp barriers when both passes are warp-local.
-template <int LOGN, int NP, int XBUF, int S0A, int HA, int S0B, int HB>
-__device__ __forceinline__ void exchange(uint32_t (&x)[NP][8], uint32_t *xb, uint32_t tau) {
-  constexpr int W = NttShape<LOGN>::XB_WORDS;
-  constexpr bool WARP = pass_warp_local<LOGN, (S0A < S0B ? S0A : S0B)>();
+template <int LOGN, int E, int NP, int XBUF, int S0A, int HA, int S0B, int HB>
+__device__ __forceinline__ void exchange(uint32_t (&x)[NP][E], uint32_t *xb, uint32_t tau) {
+  constexpr int W = NttShape<LOGN, E>::XB_WORDS;
+  constexpr bool WARP = pass_warp_local<LOGN, E, (S0A < S0B ? S0A : S0B)>();
   static_assert(XBUF == 1 || XBUF == NP, "exchange buffer must hold one or all polynomials");
   if constexpr (XBUF == NP) {
     if constexpr (WARP) __syncwarp(); else __syncthreads();
 #pragma unroll
-    for (int k = 0; k < NP; ++k) xb_store<LOGN, S0A, HA>(xb + k * W, x[k], tau);
+    for (int k = 0; k < NP; ++k) xb_store<LOGN, E, S0A, HA>(xb + k * W, x[k], tau);
     if constexpr (WARP) __syncwarp(); else __syncthreads();
 #pragma unroll
-    for (int k = 0; k < NP; ++k) xb_load<LOGN, S0B, HB>(xb + k * W, x[k], tau);
+    for (int k = 0; k < NP; ++k) xb_load<LOGN, E, S0B, HB>(xb + k * W, x[k], tau);
   } else {
 #pragma unroll
     for (int k = 0; k < NP; ++k) {
       if constexpr (WARP) __syncwarp(); else __syncthreads();
-      xb_store<LOGN, S0A, HA>(xb, x[k], tau);
+      xb_store<LOGN, E, S0A, HA>(xb, x[k], tau);
       if constexpr (WARP) __syncwarp(); else __syncthreads();
-      xb_load<LOGN, S0B, HB>(xb, x[k], tau);
+      xb_load<LOGN, E, S0B, HB>(xb, x[k], tau);
     }
   }
 }
 
 // Forward transform of NP polynomials held as x[k][e] = element
-// slot_index<LOGN,0,3>(tau, e) = tau + e*N/8 of polynomial k.
-template <int LOGN, int NP, int XBUF, int PASS = 0>
-__device__ __forceinline__ void ntt_forward(uint32_t (&x)[NP][8], const uint2 *tw, uint32_t *xb, uint32_t tau,
+// slot_index<LOGN,E,0,RAD>(tau, e) = tau + e*N/E of polynomial k.
+template <int LOGN, int E, int NP, int XBUF, int PASS = 0>
+__device__ __forceinline__ void ntt_forward(uint32_t (&x)[NP][E], const uint2 *tw, uint32_t *xb, uint32_t tau,
                                             uint32_t p) {
-  using S = NttShape<LOGN>;
-  constexpr int S0 = 3 * PASS;
+  using S = NttShape<LOGN, E>;
+  constexpr int S0 = S::RAD * PASS;
   constexpr int H = S::template h<PASS>();
-  fwd_pass<LOGN, NP, S0, H>(x, tw, tau, p, 2 * p, 4 * p);
+  fwd_pass<LOGN, E, NP, S0, H>(x, tw, tau, p, 2 * p, 4 * p);
   if constexpr (PASS + 1 < S::NPASS) {
-    exchange<LOGN, NP, XBUF, S0, H, S0 + 3, S::template h<PASS + 1>()>(x, xb, tau);
-    ntt_forward<LOGN, NP, XBUF, PASS + 1>(x, tw, xb, tau, p);
+    exchange<LOGN, E, NP, XBUF, S0, H, S0 + S::RAD, S::template h<PASS + 1>()>(x, xb, tau);
+    ntt_forward<LOGN, E, NP, XBUF, PASS + 1>(x, tw, xb, tau, p);
   }
 }
 
 // Inverse transform (without the N^{-1} factor).  Input: x[k][e] holds
-// bit-reversed position 8*tau + e; output: natural position tau + e*N/8.
-template <int LOGN, int NP, int XBUF, int PASS = NttShape<LOGN>::NPASS - 1>
-__device__ __forceinline__ void ntt_inverse(uint32_t (&x)[NP][8], const uint2 *tw, uint32_t *xb, uint32_t tau,
+// bit-reversed position E*tau + e; output: natural position tau + e*N/E.
+template <int LOGN, int E, int NP, int XBUF, int PASS = NttShape<LOGN, E>::NPASS - 1>
+__device__ __forceinline__ void ntt_inverse(uint32_t (&x)[NP][E], const uint2 *tw, uint32_t *xb, uint32_t tau,
                                             uint32_t p) {
-  using S = NttShape<LOGN>;
-  constexpr int S0 = 3 * PASS;
+  using S = NttShape<LOGN, E>;
+  constexpr int S0 = S::RAD * PASS;
   constexpr int H = S::template h<PASS>();
-  inv_pass<LOGN, NP, S0, H>(x, tw, tau, p, 4 * p);
+  inv_pass<LOGN, E, NP, S0, H>(x, tw, tau, p, 4 * p);
   if constexpr (PASS > 0) {
-    exchange<LOGN, NP, XBUF, S0, H, S0 - 3, 3>(x, xb, tau);
-    ntt_inverse<LOGN, NP, XBUF, PASS - 1>(x, tw, xb, tau, p);
+    exchange<LOGN, E, NP, XBUF, S0, H, S0 - S::RAD, S::RAD>(x, xb, tau);
+    ntt_inverse<LOGN, E, NP, XBUF, PASS - 1>(x, tw, xb, tau, p);
   }
 }
 

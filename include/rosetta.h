@@ -128,6 +128,35 @@ int rosetta_blind_rotate_extract_batch(rosetta_ctx *ctx, const uint64_t *lwe_in,
 int rosetta_keyswitch_batch(rosetta_ctx *ctx, const uint64_t *lwe_big_in, uint32_t batch,
                             uint64_t *lwe_out, void *stream);
 
+/* Many LUTs in one launch.  The paper batches independent per-element
+ * lookups (Segmented LUT Evaluation, "Multi-Value Batching"), and different
+ * nonlinear layers (softmax heads, FFN activations) can share one launch
+ * when each ciphertext names its own table: ciphertext b is bootstrapped with
+ * LUT luts[lut_index[b]].
+ *   luts      [num_luts][2^p] torus words, device memory
+ *   lut_index [batch] uint32, device memory, 4-byte aligned
+ *   lwe_in / lwe_out as for rosetta_pbs_batch (device or host)
+ * The kernel reads luts and lut_index directly.  An index >= num_luts is
+ * never followed: that ciphertext uses LUT 0 and the next
+ * rosetta_sync_status returns INVALID_ARG.  Errors: INVALID_ARG,
+ * KEYS_MISSING, CUDA, OOM. */
+int rosetta_pbs_batch_multi_lut(rosetta_ctx *ctx, const uint64_t *lwe_in, uint32_t batch, const uint64_t *luts,
+                                uint32_t num_luts, const uint32_t *lut_index, uint64_t *lwe_out, void *stream);
+
+/* Blind rotation of encrypted test polynomials.  The paper's lookup protocol
+ * (Cryptographic Lookup Protocol, Steps 2 and 3; Algorithm 1) rotates a
+ * per-element RLWE ciphertext of the table, not a public LUT: for each b,
+ *   glwe_out[b] = X^{-b~} glwe_in[b] rotated further by X^{a~_i s_i} through
+ *                 the n CMux steps, i.e. an encryption of X^{-phi~} M_b where
+ *                 glwe_in[b] encrypts M_b and phi~ = b~ - sum a~_i s_i (mod 2N)
+ *                 is the modulus-switched phase of lwe_in[b].
+ *   lwe_in  [batch][n+1], glwe_in and glwe_out [batch][k+1][N] uint64
+ *   (component-major: the k masks, then the body), all device memory.
+ * No extraction and no key switch: the result stays a GLWE ciphertext.
+ * Needs the BSK.  Errors: INVALID_ARG, KEYS_MISSING, CUDA. */
+int rosetta_blind_rotate_glwe_batch(rosetta_ctx *ctx, const uint64_t *lwe_in, uint32_t batch,
+                                    const uint64_t *glwe_in, uint64_t *glwe_out, void *stream);
+
 /* Same computation and result as rosetta_pbs_batch, for callers that cannot
  * allocate device memory during the call (their device memory belongs to
  * another allocator, or their serving loop forbids allocation after
@@ -145,7 +174,9 @@ int rosetta_pbs_batch_noalloc(rosetta_ctx *ctx, const uint64_t *lwe_in, uint32_t
                               const uint64_t *lut, uint64_t *lwe_out, void *stream);
 
 /* Wait for all work on `stream` and report any deferred execution error
- * (CUDA, TIMEOUT).  Returns OK when the stream finished cleanly. */
+ * (CUDA, TIMEOUT, or INVALID_ARG for an out-of-range LUT index seen by
+ * rosetta_pbs_batch_multi_lut; that flag is cleared once reported).  Returns
+ * OK when the stream finished cleanly. */
 int rosetta_sync_status(rosetta_ctx *ctx, void *stream);
 
 /* Free everything the context owns.  Waits for the context's device work.

@@ -78,6 +78,7 @@ def lib():
             L.orc_cmux_rotate.argtypes = [P, P, u32, u32, u32, u32, u32]
             L.orc_blind_rotate.argtypes = [P, pp, P, P, P]
             L.orc_sample_extract.argtypes = [P, P, u32, u32]
+            L.orc_blind_rotate_glwe.argtypes = [P, pp, P, P, P]
             L.orc_keyswitch.argtypes = [P, pp, P, P]
             L.orc_blind_rotate_extract.argtypes = [P, pp, P, P, P]
             L.orc_pbs.argtypes = [P, pp, P, P, P, P]
@@ -282,6 +283,35 @@ def blind_rotate(p, bsk, lwe, lut) -> np.ndarray:
     acc = np.empty((p.k + 1, p.N), np.uint64)
     L.orc_blind_rotate(_u64p(acc), ctypes.byref(P), _u64p(_c(bsk)), _u64p(_c(lwe)), _u64p(_c(lut)))
     return acc
+
+
+def blind_rotate_glwe_batch(p, bsk, lwe, glwe_in, threads=None) -> np.ndarray:
+    """[batch][(k+1)][N]: blind rotation of each ciphertext's own GLWE test
+    polynomial glwe_in[b] by the phase of lwe[b]."""
+    L = lib()
+    P = params(p)
+    lwe = _c(np.atleast_2d(lwe))
+    glwe_in = _c(glwe_in).reshape(lwe.shape[0], p.k + 1, p.N)
+    bsk = _c(bsk)
+    out = np.empty_like(glwe_in)
+
+    def one(b):
+        L.orc_blind_rotate_glwe(_u64p(out[b]), ctypes.byref(P), _u64p(bsk), _u64p(lwe[b]), _u64p(glwe_in[b]))
+
+    with ThreadPoolExecutor(threads or default_threads()) as ex:
+        list(ex.map(one, range(lwe.shape[0])))
+    return out
+
+
+def pbs_batch_multi_lut(p, bsk, ksk, lwe, luts, lut_index, threads=None) -> np.ndarray:
+    """PBS of ciphertext b with LUT luts[lut_index[b]]."""
+    lwe = _c(np.atleast_2d(lwe))
+    luts = _c(luts)
+    out = np.empty((lwe.shape[0], p.n + 1), np.uint64)
+    for li in np.unique(lut_index):
+        sel = np.nonzero(np.asarray(lut_index) == li)[0]
+        out[sel] = pbs_batch(p, bsk, ksk, lwe[sel], luts[li], threads)
+    return out
 
 
 def blind_rotate_extract_batch(p, bsk, lwe, lut, threads=None) -> np.ndarray:

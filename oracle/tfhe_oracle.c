@@ -246,6 +246,18 @@ static uint32_t log2_u32(uint32_t x) {
   return r;
 }
 
+/* The n CMux steps of blind rotation on an accumulator already initialised
+ * to X^{-b~} times the test polynomial (public or encrypted). */
+static void cmux_steps(uint64_t *acc, const orc_params *P, const uint64_t *bsk, const uint64_t *lwe,
+                       uint32_t log2_2N) {
+  const size_t ggsw_words = (size_t)(P->k + 1) * P->level * (P->k + 1) * P->N;
+  for (uint32_t i = 0; i < P->n; ++i) {
+    uint32_t a_tilde = orc_modswitch(lwe[i], log2_2N);
+    if (a_tilde == 0) continue;
+    orc_cmux_rotate(acc, bsk + i * ggsw_words, a_tilde, P->k, P->N, P->base_log, P->level);
+  }
+}
+
 /* Blind rotation: modulus-switch the LWE to Z_{2N} (a~_i, b~), start from the
  * trivial GLWE (0, X^{-b~} * v), then for i = 0..n-1 rotate by X^{a~_i s_i}
  * through the CMux with BSK_i.  The result encrypts X^{-phi~} * v with
@@ -261,12 +273,23 @@ void orc_blind_rotate(uint64_t *acc, const orc_params *P, const uint64_t *bsk,
   memset(acc, 0, sizeof(uint64_t) * (size_t)(k + 1) * N);
   uint32_t b_tilde = orc_modswitch(lwe[P->n], log2_2N);
   orc_poly_monomial(acc + (size_t)k * N, v, (2 * N - b_tilde) % (2 * N), N);
-  for (uint32_t i = 0; i < P->n; ++i) {
-    uint32_t a_tilde = orc_modswitch(lwe[i], log2_2N);
-    if (a_tilde == 0) continue;
-    orc_cmux_rotate(acc, bsk + i * ggsw_words, a_tilde, k, N, P->base_log, P->level);
-  }
+  (void)ggsw_words;
+  cmux_steps(acc, P, bsk, lwe, log2_2N);
   free(v);
+}
+
+/* Blind rotation of an encrypted test polynomial (the lookup protocol's
+ * BlindRot of a per-element RLWE ciphertext, Cryptographic Lookup Protocol
+ * Steps 2-3): the accumulator starts as X^{-b~} times the input GLWE
+ * (every component), then the same n CMux steps. */
+void orc_blind_rotate_glwe(uint64_t *acc, const orc_params *P, const uint64_t *bsk, const uint64_t *lwe,
+                           const uint64_t *glwe_in) {
+  const uint32_t N = P->N;
+  const uint32_t log2_2N = log2_u32(2 * N);
+  const uint32_t b_tilde = orc_modswitch(lwe[P->n], log2_2N);
+  for (uint32_t c = 0; c <= P->k; ++c)
+    orc_poly_monomial(acc + (size_t)c * N, glwe_in + (size_t)c * N, (2 * N - b_tilde) % (2 * N), N);
+  cmux_steps(acc, P, bsk, lwe, log2_2N);
 }
 
 /* Sample extraction of the constant coefficient (Background, "LWE Extract"):

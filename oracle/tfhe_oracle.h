@@ -69,6 +69,8 @@ void orc_cmux_rotate(uint64_t *acc, const uint64_t *ggsw, uint32_t a_tilde,
                      uint32_t k, uint32_t N, uint32_t base_log, uint32_t level);
 void orc_blind_rotate(uint64_t *acc, const orc_params *P, const uint64_t *bsk,
                       const uint64_t *lwe, const uint64_t *lut);
+void orc_blind_rotate_glwe(uint64_t *acc, const orc_params *P, const uint64_t *bsk,
+                           const uint64_t *lwe, const uint64_t *glwe_in);
 void orc_sample_extract(uint64_t *lwe_big, const uint64_t *glwe, uint32_t k, uint32_t N);
 void orc_keyswitch(uint64_t *out, const orc_params *P, const uint64_t *ksk, const uint64_t *lwe_big);
 void orc_blind_rotate_extract(uint64_t *lwe_big, const orc_params *P, const uint64_t *bsk,

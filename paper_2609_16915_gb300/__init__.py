@@ -21,7 +21,8 @@ STATUS = {0: "ok", -1: "invalid argument", -2: "unsupported parameters", -3: "ke
           -4: "CUDA error", -5: "out of device memory", -6: "device wait timed out"}
 
 EXPORTS = ("rosetta_params_init", "rosetta_upload_bsk", "rosetta_upload_ksk", "rosetta_pbs_batch",
-           "rosetta_blind_rotate_extract_batch", "rosetta_keyswitch_batch", "rosetta_pbs_batch_noalloc",
+           "rosetta_blind_rotate_extract_batch", "rosetta_keyswitch_batch", "rosetta_pbs_batch_multi_lut",
+           "rosetta_blind_rotate_glwe_batch", "rosetta_pbs_batch_noalloc",
            "rosetta_sync_status", "rosetta_destroy", "rosetta_status_string")
 
 
@@ -56,6 +57,8 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     L.rosetta_blind_rotate_extract_batch.argtypes = [vp, u64p, u32, u64p, u64p, vp]
     L.rosetta_keyswitch_batch.argtypes = [vp, u64p, u32, u64p, vp]
     L.rosetta_pbs_batch_noalloc.argtypes = [vp, u64p, u32, u64p, u64p, vp]
+    L.rosetta_pbs_batch_multi_lut.argtypes = [vp, u64p, u32, u64p, u32, vp, u64p, vp]
+    L.rosetta_blind_rotate_glwe_batch.argtypes = [vp, u64p, u32, u64p, u64p, vp]
     L.rosetta_sync_status.argtypes = [vp, vp]
     L.rosetta_destroy.argtypes = [vp]
     L.rosetta_destroy.restype = None
@@ -158,6 +161,22 @@ class Context:
                                                                          _ptr(lwe_out), _stream(stream)))
         return lwe_out
 
+    def rosetta_pbs_batch_multi_lut(self, lwe_in, luts, lut_index, lwe_out, stream=None):
+        """PBS with a LUT per ciphertext: luts [num_luts][2^p], lut_index [batch] (uint32 / int32 tensor)."""
+        batch = lwe_in.shape[0]
+        _check("rosetta_pbs_batch_multi_lut",
+               load().rosetta_pbs_batch_multi_lut(self._h, _ptr(lwe_in), batch, _ptr(luts), luts.shape[0],
+                                                  _ptr(lut_index), _ptr(lwe_out), _stream(stream)))
+        return lwe_out
+
+    def rosetta_blind_rotate_glwe_batch(self, lwe_in, glwe_in, glwe_out, stream=None):
+        """Blind rotation of per-ciphertext GLWE test polynomials [batch][k+1][N]."""
+        batch = lwe_in.shape[0]
+        _check("rosetta_blind_rotate_glwe_batch",
+               load().rosetta_blind_rotate_glwe_batch(self._h, _ptr(lwe_in), batch, _ptr(glwe_in), _ptr(glwe_out),
+                                                      _stream(stream)))
+        return glwe_out
+
     def rosetta_pbs_batch_noalloc(self, lwe_in, lut, lwe_out, stream=None):
         """rosetta_pbs_batch without any device allocation in the call (fixed
         in-library scratch; device buffers only, bounded batch)."""
@@ -175,4 +194,6 @@ class Context:
     pbs_batch = rosetta_pbs_batch
     blind_rotate_extract_batch = rosetta_blind_rotate_extract_batch
     keyswitch_batch = rosetta_keyswitch_batch
+    pbs_batch_multi_lut = rosetta_pbs_batch_multi_lut
+    blind_rotate_glwe_batch = rosetta_blind_rotate_glwe_batch
     sync_status = rosetta_sync_status

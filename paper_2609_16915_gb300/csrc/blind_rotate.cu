@@ -99,19 +99,42 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
   __syncthreads();
   {
     const uint32_t btil = atil[a.n];
-    const uint32_t box = N >> a.msg_bits, h = box >> 1;
+    if (a.glwe_in) {
+      // encrypted test polynomial: ACC = X^{-b~} (A, B) for this ciphertext
+      const uint64_t *gin = a.glwe_in + static_cast<size_t>(ct) * 2 * N;
 #pragma unroll
-    for (int m = 0; m < ITEMS; ++m) {
-      const uint32_t item = tau + m * T;
-      const uint32_t c = item / Q, jl = item % Q, j = rank * Q + jl;
-      if (c == 0) {
-        acc[jl] = 0;
-      } else {
-        // (X^{2N - b~} v)[j] = +-v[t], t = (j + b~) mod 2N folded into [0, N)
+      for (int m = 0; m < ITEMS; ++m) {
+        const uint32_t item = tau + m * T;
+        const uint32_t c = item / Q, jl = item % Q, j = rank * Q + jl;
         const uint32_t e = (j + btil) & (TWO_N - 1);
-        const uint32_t t = e & (N - 1);
-        const uint64_t v = (t < N - h) ? a.lut[(t + h) / box] : (0ull - a.lut[0]);
-        acc[Q + jl] = (e >= N) ? 0ull - v : v;
+        const uint64_t v = gin[c * N + (e & (N - 1))];
+        acc[c * Q + jl] = (e >= N) ? 0ull - v : v;
+      }
+    } else {
+      // trivial GLWE (0, X^{-b~} v) of the test polynomial of this ciphertext's LUT
+      uint32_t li = 0;
+      if (a.lut_index) {
+        li = a.lut_index[ct];
+        if (li >= a.num_luts) {  // never read outside the LUT array
+          if (tau == 0 && rank == 0 && a.err_flag) atomicExch(a.err_flag, 1u);
+          li = 0;
+        }
+      }
+      const uint64_t *lut = a.lut + (static_cast<size_t>(li) << a.msg_bits);
+      const uint32_t box = N >> a.msg_bits, h = box >> 1;
+#pragma unroll
+      for (int m = 0; m < ITEMS; ++m) {
+        const uint32_t item = tau + m * T;
+        const uint32_t c = item / Q, jl = item % Q, j = rank * Q + jl;
+        if (c == 0) {
+          acc[jl] = 0;
+        } else {
+          // (X^{2N - b~} v)[j] = +-v[t], t = (j + b~) mod 2N folded into [0, N)
+          const uint32_t e = (j + btil) & (TWO_N - 1);
+          const uint32_t t = e & (N - 1);
+          const uint64_t v = (t < N - h) ? lut[(t + h) / box] : (0ull - lut[0]);
+          acc[Q + jl] = (e >= N) ? 0ull - v : v;
+        }
       }
     }
   }
@@ -235,16 +258,27 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
     cluster.sync();
   }
 
-  // ---- sample extraction of the constant coefficient ----
-  uint64_t *out = a.lwe_big_out + static_cast<size_t>(ct) * (N + 1);
+  if (a.glwe_out) {
+    // ---- the rotated accumulator itself ----
+    uint64_t *gout = a.glwe_out + static_cast<size_t>(ct) * 2 * N;
 #pragma unroll
-  for (int m = 0; m < ITEMS; ++m) {
-    const uint32_t item = tau + m * T;
-    const uint32_t c = item / Q, jl = item % Q, j = rank * Q + jl;
-    if (c == 0) {
-      out[j == 0 ? 0 : N - j] = (j == 0) ? acc[jl] : 0ull - acc[jl];
-    } else if (j == 0) {
-      out[N] = acc[Q];
+    for (int m = 0; m < ITEMS; ++m) {
+      const uint32_t item = tau + m * T;
+      const uint32_t c = item / Q, jl = item % Q;
+      gout[c * N + rank * Q + jl] = acc[c * Q + jl];
+    }
+  } else {
+    // ---- sample extraction of the constant coefficient ----
+    uint64_t *out = a.lwe_big_out + static_cast<size_t>(ct) * (N + 1);
+#pragma unroll
+    for (int m = 0; m < ITEMS; ++m) {
+      const uint32_t item = tau + m * T;
+      const uint32_t c = item / Q, jl = item % Q, j = rank * Q + jl;
+      if (c == 0) {
+        out[j == 0 ? 0 : N - j] = (j == 0) ? acc[jl] : 0ull - acc[jl];
+      } else if (j == 0) {
+        out[N] = acc[Q];
+      }
     }
   }
   cluster.sync();

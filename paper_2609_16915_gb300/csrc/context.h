@@ -27,4 +27,5 @@ struct rosetta_ctx {
   uint64_t *d_out = nullptr;      // staging for host outputs
   size_t out_words_cap = 0;
   uint64_t *d_lut = nullptr;      // staging for a host LUT  [2^p]
+  uint32_t *d_err = nullptr;      // device-side argument error flag (LUT index out of range)
 };

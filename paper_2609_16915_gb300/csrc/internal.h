@@ -33,11 +33,15 @@ struct CrtConsts {
 
 struct BrArgs {
   const uint64_t *lwe_in;   // [batch][n+1]
-  const uint64_t *lut;      // [2^p]
-  uint64_t *lwe_big_out;    // [batch][N+1]   (k = 1)
+  const uint64_t *lut;      // [num_luts][2^p]; ignored when glwe_in is set
+  uint64_t *lwe_big_out;    // [batch][N+1] extracted LWEs (k = 1), or
+  uint64_t *glwe_out;       // [batch][2][N] rotated accumulators (when set)
+  const uint32_t *lut_index;  // [batch] LUT of each ciphertext, or null (LUT 0)
+  const uint64_t *glwe_in;  // [batch][2][N] GLWE test polynomials, or null
+  uint32_t *err_flag;       // set to 1 when a LUT index is out of range
   const uint32_t *bsk;      // transform domain [n][prime][2l][2][N]
   const uint2 *tw;          // [prime][N] (W, Shoup companion)
-  uint32_t n, level, base_log, msg_bits, batch;
+  uint32_t n, level, base_log, msg_bits, batch, num_luts;
   CrtConsts cc;
 };
 

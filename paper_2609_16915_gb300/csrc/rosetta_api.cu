@@ -164,6 +164,8 @@ BrArgs br_args(const rosetta_ctx *c, const uint64_t *in, uint32_t batch, const u
   a.base_log = c->prm.pbs_base_log;
   a.msg_bits = c->prm.msg_bits;
   a.batch = batch;
+  a.num_luts = 1;
+  a.err_flag = c->d_err;
   a.cc = c->cc;
   return a;
 }
@@ -231,6 +233,8 @@ int rosetta_params_init(rosetta_ctx **out, const rosetta_params *p, int cuda_dev
   cudaError_t e = cudaMalloc(&c->d_tw, tw.size() * sizeof(uint2));
   if (e == cudaSuccess) e = cudaMemcpy(c->d_tw, tw.data(), tw.size() * sizeof(uint2), cudaMemcpyHostToDevice);
   if (e == cudaSuccess) e = cudaMalloc(&c->d_lut, sizeof(uint64_t) << p->msg_bits);
+  if (e == cudaSuccess) e = cudaMalloc(&c->d_err, sizeof(uint32_t));
+  if (e == cudaSuccess) e = cudaMemset(c->d_err, 0, sizeof(uint32_t));
   if (e != cudaSuccess) {
     rosetta_destroy(c);
     return cuda_fail(e);
@@ -361,12 +365,66 @@ int rosetta_pbs_batch(rosetta_ctx *c, const uint64_t *lwe_in, uint32_t batch, co
   return finish_io(c, lwe_out, lwe_words(c), batch, st, s);
 }
 
+int rosetta_pbs_batch_multi_lut(rosetta_ctx *c, const uint64_t *lwe_in, uint32_t batch, const uint64_t *luts,
+                                uint32_t num_luts, const uint32_t *lut_index, uint64_t *lwe_out, void *stream) {
+  if (!c) return ROSETTA_ERR_INVALID_ARG;
+  if (batch == 0) return ROSETTA_OK;
+  if (!lwe_in || !luts || !lut_index || !lwe_out || num_luts == 0) return ROSETTA_ERR_INVALID_ARG;
+  if (!c->have_bsk || !c->have_ksk) return ROSETTA_ERR_KEYS_MISSING;
+  if (cudaSetDevice(c->device) != cudaSuccess) return ROSETTA_ERR_CUDA;
+  // the LUT table and the index array are read by the kernel directly
+  if (!is_device_ptr(luts) || !is_device_ptr(lut_index) || !aligned8(luts) ||
+      (reinterpret_cast<uintptr_t>(lut_index) & 3u))
+    return ROSETTA_ERR_INVALID_ARG;
+  cudaStream_t s = as_stream(stream);
+  Staged st;
+  int r = stage_io(c, lwe_in, lwe_words(c), batch, nullptr, lwe_out, lwe_words(c), s, &st);
+  if (r != ROSETTA_OK) return r;
+  r = ensure_big(c, batch, s);
+  if (r != ROSETTA_OK) return r;
+  BrArgs a = br_args(c, st.in, batch, luts, c->d_big);
+  a.lut_index = lut_index;
+  a.num_luts = num_luts;
+  cudaError_t e = launch_blind_rotate(a, c->logN, c->dig16, s);
+  if (e != cudaSuccess) return cuda_fail(e);
+  e = launch_keyswitch(ks_args(c, c->d_big, batch, st.out), s);
+  if (e != cudaSuccess) return cuda_fail(e);
+  return finish_io(c, lwe_out, lwe_words(c), batch, st, s);
+}
+
+int rosetta_blind_rotate_glwe_batch(rosetta_ctx *c, const uint64_t *lwe_in, uint32_t batch, const uint64_t *glwe_in,
+                                    uint64_t *glwe_out, void *stream) {
+  if (!c) return ROSETTA_ERR_INVALID_ARG;
+  if (batch == 0) return ROSETTA_OK;
+  if (!lwe_in || !glwe_in || !glwe_out) return ROSETTA_ERR_INVALID_ARG;
+  if (!c->have_bsk) return ROSETTA_ERR_KEYS_MISSING;
+  if (cudaSetDevice(c->device) != cudaSuccess) return ROSETTA_ERR_CUDA;
+  const size_t gw = 2 * (size_t)c->prm.poly_size;
+  if (!is_device_ptr(lwe_in) || !is_device_ptr(glwe_in) || !is_device_ptr(glwe_out) || !aligned8(lwe_in) ||
+      !aligned8(glwe_in) || !aligned8(glwe_out))
+    return ROSETTA_ERR_INVALID_ARG;
+  const size_t gbytes = (size_t)batch * gw * 8;
+  if (overlaps(glwe_in, gbytes, glwe_out, gbytes) || overlaps(lwe_in, (size_t)batch * lwe_words(c) * 8, glwe_out, gbytes))
+    return ROSETTA_ERR_INVALID_ARG;
+  BrArgs a = br_args(c, lwe_in, batch, nullptr, nullptr);
+  a.glwe_in = glwe_in;
+  a.glwe_out = glwe_out;
+  cudaError_t e = launch_blind_rotate(a, c->logN, c->dig16, as_stream(stream));
+  return e == cudaSuccess ? ROSETTA_OK : cuda_fail(e);
+}
+
 int rosetta_sync_status(rosetta_ctx *c, void *stream) {
   if (!c) return ROSETTA_ERR_INVALID_ARG;
   if (cudaSetDevice(c->device) != cudaSuccess) return ROSETTA_ERR_CUDA;
   cudaError_t e = cudaStreamSynchronize(as_stream(stream));
   if (e == cudaSuccess) e = cudaGetLastError();
-  return e == cudaSuccess ? ROSETTA_OK : cuda_fail(e);
+  if (e != cudaSuccess) return cuda_fail(e);
+  // an out-of-range LUT index seen by a kernel is reported once, then cleared
+  uint32_t flag = 0;
+  e = cudaMemcpy(&flag, c->d_err, sizeof(flag), cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess && flag) e = cudaMemset(c->d_err, 0, sizeof(flag));
+  if (e != cudaSuccess) return cuda_fail(e);
+  return flag ? ROSETTA_ERR_INVALID_ARG : ROSETTA_OK;
 }
 
 void rosetta_destroy(rosetta_ctx *c) {
@@ -381,6 +439,7 @@ void rosetta_destroy(rosetta_ctx *c) {
   cudaFree(c->d_in);
   cudaFree(c->d_out);
   cudaFree(c->d_lut);
+  cudaFree(c->d_err);
   delete c;
 }
 

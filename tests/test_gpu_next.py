@@ -1,0 +1,111 @@
+"""GPU parity of the widened entry points: a LUT per ciphertext (many LUTs
+in one launch) and blind rotation of encrypted (GLWE) test polynomials.
+Bit-exact against the CPU oracle."""
+
+import numpy as np
+import pytest
+
+import oracle as O
+import workload as W
+from tests import gpu_util as G
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2609_16915_gb300 import build
+    build.build()
+
+
+def _index_dev(idx):
+    import torch
+    return torch.from_numpy(np.asarray(idx, dtype=np.int32)).cuda()
+
+
+def test_multi_lut_bitexact_and_decrypts():
+    p = W.CONFIGS["tiny"]
+    keys = O.Keys(p, W.key_draws(p))
+    tables = [[(m * m) % 8 for m in range(8)], [(3 * m + 1) % 8 for m in range(8)], [7 - m for m in range(8)]]
+    luts = np.stack([W.lut_torus(p, codes=t) for t in tables])
+    rs = np.random.default_rng(2)
+    idx = rs.integers(0, 3, size=40)
+    cd = W.cipher_draws(p, 40, sub=21)
+    lwe = keys.encrypt(cd)
+    ctx = G.make_ctx(p, keys.bsk, keys.ksk)
+    out = G.empty_dev(40, p.n + 1)
+    ctx.pbs_batch_multi_lut(G.to_dev(lwe), G.to_dev(luts), _index_dev(idx), out)
+    ctx.sync_status()
+    got = G.to_host(out)
+    assert np.array_equal(got, O.pbs_batch_multi_lut(p, keys.bsk, keys.ksk, lwe, luts, idx))
+    want_codes = np.array([tables[i][m] for i, m in zip(idx, cd.codes)])
+    assert np.array_equal(keys.decrypt(got), want_codes)
+
+
+def test_multi_lut_bad_index_is_reported_not_followed():
+    import paper_2609_16915_gb300 as R
+    p = W.CONFIGS["tiny"]
+    keys = O.Keys(p, W.key_draws(p))
+    luts = np.stack([W.lut_torus(p), W.lut_torus(p, codes=[1] * 8)])
+    lwe = W.uniform_ciphertexts(p, 4, sub=22)
+    ctx = G.make_ctx(p, keys.bsk, keys.ksk)
+    out = G.empty_dev(4, p.n + 1)
+    ctx.pbs_batch_multi_lut(G.to_dev(lwe), G.to_dev(luts), _index_dev([0, 1, 5, 1]), out)
+    with pytest.raises(R.RosettaError) as e:
+        ctx.sync_status()
+    assert e.value.status == -1
+    ctx.sync_status()                                   # the flag is cleared once reported
+    got = G.to_host(out)
+    want = O.pbs_batch_multi_lut(p, keys.bsk, keys.ksk, lwe, luts, [0, 1, 0, 1])
+    assert np.array_equal(got, want)
+
+
+@pytest.mark.parametrize("name", ["tiny", "standard"])
+def test_glwe_blind_rotation_bitexact(name):
+    p = W.CONFIGS[name]
+    if name == "tiny":
+        keys = O.Keys(p, W.key_draws(p))
+        bsk, ksk = keys.bsk, keys.ksk
+        lwe = keys.encrypt(W.cipher_draws(p, 9, sub=23))
+    else:
+        bsk, ksk = W.uniform_keys(p, seed=31)
+        lwe = G.sparse_lwe(p, 3, 2, seed=4)
+    glwe = W.uniform_u64((lwe.shape[0], p.k + 1, p.N), W.rng(p.seed, "sample", 24))
+    ctx = G.make_ctx(p, bsk, ksk)
+    out = G.empty_dev(lwe.shape[0], p.k + 1, p.N)
+    ctx.blind_rotate_glwe_batch(G.to_dev(lwe), G.to_dev(glwe), out)
+    ctx.sync_status()
+    assert np.array_equal(G.to_host(out), O.blind_rotate_glwe_batch(p, bsk, lwe, glwe))
+
+
+def test_glwe_blind_rotation_trivial_input_matches_pbs_path():
+    """A trivial GLWE of the test polynomial through the GLWE entry point,
+    then extraction and key switch, gives rosetta_pbs_batch's words."""
+    p = W.CONFIGS["standard"]
+    bsk, ksk = W.uniform_keys(p, seed=32)
+    lwe = G.sparse_lwe(p, 2, 3, seed=6)
+    lut = W.lut_torus(p)
+    glwe = np.zeros((2, p.k + 1, p.N), np.uint64)
+    glwe[:, p.k] = O.test_poly(lut, p.msg_bits, p.N)
+    ctx = G.make_ctx(p, bsk, ksk)
+    out = G.empty_dev(2, p.k + 1, p.N)
+    ctx.blind_rotate_glwe_batch(G.to_dev(lwe), G.to_dev(glwe), out)
+    ctx.sync_status()
+    acc = G.to_host(out)
+    big = np.stack([O.sample_extract(acc[b]) for b in range(2)])
+    assert np.array_equal(G.gpu_keyswitch(ctx, p, big), G.gpu_pbs(ctx, p, lwe, lut))
+
+
+def test_glwe_blind_rotation_rejects_host_buffers():
+    import paper_2609_16915_gb300 as R
+    p = W.CONFIGS["tiny"]
+    keys = O.Keys(p, W.key_draws(p))
+    ctx = G.make_ctx(p, keys.bsk, keys.ksk)
+    lwe = W.uniform_ciphertexts(p, 2)
+    glwe = np.zeros((2, p.k + 1, p.N), np.uint64)
+    with pytest.raises(R.RosettaError) as e:
+        ctx.blind_rotate_glwe_batch(lwe, glwe, np.zeros_like(glwe))
+    assert e.value.status == -1

@@ -316,3 +316,59 @@ def test_keyswitch_noiseless_key_closed_form():
         want = (int(big[b, -1]) - sum(int(keys.big_key[i]) * _round_top(int(big[b, i]), bits)
                                       for i in range(p.kN))) % Q
         assert int(out[b, -1]) == want
+
+
+# ------------------------------------------------------------------ blind rotation of an encrypted test polynomial
+
+def test_glwe_blind_rotation_of_trivial_glwe_is_the_lut_path():
+    """Rotating the trivial GLWE (0, v) must reproduce the public-LUT blind
+    rotation word for word."""
+    p = W.CONFIGS["tiny"]
+    keys = O.Keys(p, W.key_draws(p))
+    lut = W.lut_torus(p)
+    v = O.test_poly(lut, p.msg_bits, p.N)
+    lwe = W.uniform_ciphertexts(p, 3, sub=11)
+    glwe = np.zeros((3, p.k + 1, p.N), np.uint64)
+    glwe[:, p.k] = v
+    got = O.blind_rotate_glwe_batch(p, keys.bsk, lwe, glwe)
+    for b in range(3):
+        assert np.array_equal(got[b], O.blind_rotate(p, keys.bsk, lwe[b], lut))
+
+
+def test_glwe_blind_rotation_noiseless_closed_form():
+    """With noiseless keys and input words that are multiples of 2^(64 -
+    base_log*level) (so the gadget rounding is exact), the output is exactly
+    X^{-phi~} times the input GLWE, phi~ the modulus-switched phase."""
+    p = W.CONFIGS["tiny"]
+    keys = O.Keys(p, W.key_draws(p, trivial=True))
+    rs = np.random.default_rng(8)
+    shift = np.uint64(64 - p.pbs_base_log * p.pbs_level)
+    glwe = (rs.integers(0, 2**63, size=(4, p.k + 1, p.N), dtype=np.uint64) << shift).astype(np.uint64)
+    lwe = W.uniform_ciphertexts(p, 4, sub=12)
+    got = O.blind_rotate_glwe_batch(p, keys.bsk, lwe, glwe)
+    two_n = 2 * p.N
+    for b in range(4):
+        ms = [((2 * int(x) * two_n + Q) // (2 * Q)) % two_n for x in lwe[b]]
+        phi = (ms[-1] - sum(ms[i] * int(keys.lwe_key[i]) for i in range(p.n))) % two_n
+        for c in range(p.k + 1):
+            assert np.array_equal(got[b, c], O.poly_monomial(glwe[b, c], (two_n - phi) % two_n))
+
+
+def test_glwe_blind_rotation_decrypts_to_rotated_table():
+    """Real keys, an encrypted test polynomial: the GLWE phase of the output
+    holds the table rotated left by the encrypted message (its constant
+    coefficient decodes to LUT(m))."""
+    p = W.CONFIGS["tiny"]
+    keys = O.Keys(p, W.key_draws(p))
+    codes = np.arange(8)
+    cts = keys.encrypt(W.cipher_draws(p, 8, codes=codes, sub=13))
+    lut = W.lut_torus(p)
+    v = O.test_poly(lut, p.msg_bits, p.N)
+    g = W.rng(p.seed, "sample", 13)
+    glwe = np.stack([O.glwe_encrypt(keys.glwe_key, v, W.uniform_u64((p.k, p.N), g),
+                                    W.gaussian_u64((p.N,), p.glwe_sigma_log2, g)) for _ in range(8)])
+    out = O.blind_rotate_glwe_batch(p, keys.bsk, cts, glwe)
+    sh = 63 - p.msg_bits
+    for b in range(8):
+        ph = int(O.glwe_phase(keys.glwe_key, out[b])[0])
+        assert ((ph + (1 << (sh - 1))) >> sh) % (1 << (p.msg_bits + 1)) == W.lut_codes(p)[codes[b]]

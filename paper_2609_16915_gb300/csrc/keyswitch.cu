@@ -3,7 +3,9 @@
 // with d the signed base-2^beta digits of a'_i rounded to its top beta*l bits.
 //
 // This is a batched integer matrix product [batch x kN*l] digits times
-// [kN*l x (n+1)] key words.  Digits are shifted to d + B/2 in [0, B) so every
+// [kN*l x (n+1)] key words.  Small batches split the kN input words over
+// several CTAs (split-K); the partial sums are combined with 64-bit atomic
+// adds, which are exact and order-independent mod 2^64.  Digits are shifted to d + B/2 in [0, B) so every
 // product is an unsigned 32x64-bit multiply; the shift is undone with the
 // precomputed column sums corr[o] = (B/2) sum_rows KSK[row][o].  Each product
 // d * g mod 2^64 is split as d*g_lo (64-bit accumulator) + 2^32 (d*g_hi)
@@ -43,7 +45,12 @@ __global__ void __launch_bounds__(KS_THREADS) keyswitch_kernel(const KsArgs a) {
     }
 
   const uint32_t krows = KS_KI * level;
-  for (uint32_t i0 = 0; i0 < a.kN; i0 += KS_KI) {
+  // this CTA's share of the input words: [i_begin, i_end), KS_KI-aligned
+  const uint32_t chunks = (a.kN + KS_KI - 1) / KS_KI;
+  const uint32_t per = (chunks + gridDim.z - 1) / gridDim.z;
+  const uint32_t i_begin = blockIdx.z * per * KS_KI;
+  const uint32_t i_end = min(a.kN, i_begin + per * KS_KI);
+  for (uint32_t i0 = i_begin; i0 < i_end; i0 += KS_KI) {
     __syncthreads();
     for (uint32_t idx = tid; idx < KS_BM * KS_KI; idx += KS_THREADS) {
       const uint32_t ii = idx % KS_KI, m = idx / KS_KI;  // consecutive words of one ciphertext
@@ -90,8 +97,16 @@ __global__ void __launch_bounds__(KS_THREADS) keyswitch_kernel(const KsArgs a) {
       const uint32_t o = o0 + tx * KS_TN + t;
       if (o >= n1) continue;
       const uint64_t sum = lo[m][t] + (static_cast<uint64_t>(hi[m][t]) << 32);
-      const uint64_t body = (o == a.n) ? a.big[static_cast<size_t>(b) * stride_in + a.kN] : 0;
-      a.out[static_cast<size_t>(b) * n1 + o] = body - sum + a.corr[o];
+      if (gridDim.z == 1) {
+        const uint64_t body = (o == a.n) ? a.big[static_cast<size_t>(b) * stride_in + a.kN] : 0;
+        a.out[static_cast<size_t>(b) * n1 + o] = body - sum + a.corr[o];
+      } else {
+        // the output was zeroed; split 0 also adds the body and the correction
+        uint64_t v = 0ull - sum;
+        if (blockIdx.z == 0) v += ((o == a.n) ? a.big[static_cast<size_t>(b) * stride_in + a.kN] : 0) + a.corr[o];
+        atomicAdd(reinterpret_cast<unsigned long long *>(a.out + static_cast<size_t>(b) * n1 + o),
+                  static_cast<unsigned long long>(v));
+      }
     }
   }
 }
@@ -102,6 +117,21 @@ cudaError_t launch_keyswitch(const KsArgs &a, cudaStream_t s) {
       cudaFuncSetAttribute(keyswitch_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
   dim3 grid((a.n + 1 + KS_BN - 1) / KS_BN, (a.batch + KS_BM - 1) / KS_BM, 1);
+  // enough CTAs to keep every SM streaming key words: split the input words
+  // when the output tiles alone give fewer than ~4 CTAs per SM
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const uint32_t tiles = grid.x * grid.y, want = 4u * static_cast<uint32_t>(sms > 0 ? sms : 1);
+  const uint32_t chunks = (a.kN + KS_KI - 1) / KS_KI;
+  uint32_t splits = tiles >= want ? 1u : (want + tiles - 1) / tiles;
+  if (splits > chunks) splits = chunks;
+  splits = (chunks + (chunks + splits - 1) / splits - 1) / ((chunks + splits - 1) / splits);  // no empty splits
+  if (splits > 1) {
+    grid.z = splits;
+    e = cudaMemsetAsync(a.out, 0, static_cast<size_t>(a.batch) * (a.n + 1) * sizeof(uint64_t), s);
+    if (e != cudaSuccess) return e;
+  }
   keyswitch_kernel<<<grid, KS_THREADS, smem, s>>>(a);
   return cudaGetLastError();
 }

@@ -217,12 +217,26 @@ __device__ __forceinline__ void inv_pass(uint32_t (&x)[NP][E], const uint2 *tw, 
   if constexpr (U > 0) inv_pass<LOGN, E, NP, S0, H, U - 1>(x, tw, tau, p, four_p);
 }
 
-// A pass whose butterfly groups span at most 32 E elements keeps every
-// warp's 32 x E values inside one aligned range of that size, so an exchange
-// between two such passes only needs the warp to synchronise.
+// A pass whose butterfly groups span S elements keeps the data of every run of
+// G = max(1, S / (32 E)) consecutive warps inside one aligned range of 32 E G
+// elements, so an exchange out of (or into) that pass only has to
+// synchronise those G warps: the warp itself when S <= 32 E, a named barrier
+// over 32 G threads in between, the whole CTA when G covers it.
 template <int LOGN, int E, int S0>
-__host__ __device__ constexpr bool pass_warp_local() {
-  return (1 << (LOGN - S0)) <= 32 * E;
+__host__ __device__ constexpr int pass_group_warps() {
+  return (1 << (LOGN - S0)) <= 32 * E ? 1 : (1 << (LOGN - S0)) / (32 * E);
+}
+
+template <int G, int WARPS>
+__device__ __forceinline__ void group_sync(uint32_t tau) {
+  if constexpr (G <= 1) {
+    __syncwarp();
+  } else if constexpr (G >= WARPS) {
+    __syncthreads();
+  } else {
+    static_assert(WARPS / G <= 15, "named barriers 1..15");
+    asm volatile("bar.sync %0, %1;" ::"r"(1u + (tau >> 5) / G), "r"(32 * G) : "memory");
+  }
 }
 
 // Padded address of slot e of thread tau in the pass (S0, H), split as a
@@ -284,26 +298,27 @@ __device__ __forceinline__ void xb_load(const uint32_t *buf, uint32_t (&v)[E], u
 
 // Move NP register sets from the layout of pass A to that of pass B through
 // the exchange buffer xb (XBUF polynomials of NttShape::XB_WORDS words each).
-// The leading barrier protects xb from readers of the previous exchange; it
-// and the middle one are warp barriers when both passes are warp-local.
+// The leading barrier protects xb from readers of the previous exchange; both
+// barriers cover only the warps whose data the exchange mixes.
 template <int LOGN, int E, int NP, int XBUF, int S0A, int HA, int S0B, int HB>
 __device__ __forceinline__ void exchange(uint32_t (&x)[NP][E], uint32_t *xb, uint32_t tau) {
   constexpr int W = NttShape<LOGN, E>::XB_WORDS;
-  constexpr bool WARP = pass_warp_local<LOGN, E, (S0A < S0B ? S0A : S0B)>();
+  constexpr int G = pass_group_warps<LOGN, E, (S0A < S0B ? S0A : S0B)>();
+  constexpr int WARPS = NttShape<LOGN, E>::T / 32 > 0 ? NttShape<LOGN, E>::T / 32 : 1;
   static_assert(XBUF == 1 || XBUF == NP, "exchange buffer must hold one or all polynomials");
   if constexpr (XBUF == NP) {
-    if constexpr (WARP) __syncwarp(); else __syncthreads();
+    group_sync<G, WARPS>(tau);
 #pragma unroll
     for (int k = 0; k < NP; ++k) xb_store<LOGN, E, S0A, HA>(xb + k * W, x[k], tau);
-    if constexpr (WARP) __syncwarp(); else __syncthreads();
+    group_sync<G, WARPS>(tau);
 #pragma unroll
     for (int k = 0; k < NP; ++k) xb_load<LOGN, E, S0B, HB>(xb + k * W, x[k], tau);
   } else {
 #pragma unroll
     for (int k = 0; k < NP; ++k) {
-      if constexpr (WARP) __syncwarp(); else __syncthreads();
+      group_sync<G, WARPS>(tau);
       xb_store<LOGN, E, S0A, HA>(xb, x[k], tau);
-      if constexpr (WARP) __syncwarp(); else __syncthreads();
+      group_sync<G, WARPS>(tau);
       xb_load<LOGN, E, S0B, HB>(xb, x[k], tau);
     }
   }

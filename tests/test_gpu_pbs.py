@@ -159,6 +159,24 @@ def test_exp_sweep_batches(batch):
     assert fails <= max(2, batch // 100)
 
 
+@pytest.mark.parametrize("batch", [16384, 65536])
+def test_exp_sweep_large_batches_sampled(batch):
+    """The sweep's two largest launches: a seeded sample word for word, the
+    whole batch by decryption (the 5-bit exp LUT's thin margin allows a few
+    failures)."""
+    p = W.CONFIGS["exp_sweep"]
+    keys = real_keys("exp_sweep")
+    cd = W.cipher_draws(p, batch, sub=batch)
+    lwe = keys.encrypt(cd)
+    lut = W.lut_torus(p)
+    ctx = G.make_ctx(p, keys.bsk, keys.ksk, max_batch=batch)
+    got = G.gpu_pbs(ctx, p, lwe, lut)
+    sample = np.array([0, batch // 2, batch - 1])
+    assert np.array_equal(got[sample], O.pbs_batch(p, keys.bsk, keys.ksk, lwe[sample], lut))
+    fails = int(np.sum(keys.decrypt(got) != W.lut_codes(p)[cd.codes]))
+    assert fails <= batch // 100
+
+
 @pytest.mark.parametrize("name", ["gpt2_mlp", "llama_silu"])
 def test_large_configs_full_batch_sparse_sample(name):
     """Full-size launches of the two large parameter sets with uniform-word

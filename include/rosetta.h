@@ -157,6 +157,30 @@ int rosetta_pbs_batch_multi_lut(rosetta_ctx *ctx, const uint64_t *lwe_in, uint32
 int rosetta_blind_rotate_glwe_batch(rosetta_ctx *ctx, const uint64_t *lwe_in, uint32_t batch,
                                     const uint64_t *glwe_in, uint64_t *glwe_out, void *stream);
 
+/* Upload the automorphism keys of the RLWE trace (k = 1, N <= 4096).  The
+ * paper isolates the constant coefficient of an RLWE ciphertext with a trace
+ * (Background, "Scheme Conversion and Other Primitives", RLWE Trace
+ * Computation), applied after each blind rotation of its lookup protocol.
+ * Step s = 0 .. log2 N - 1 uses X -> X^k, k = 2^(log2 N - s) + 1, and key s:
+ * `level` GLWE encryptions under S of sigma_k(S) * 2^(64 - lev*base_log).
+ * Raw layout [log2 N][level][2][N] (n_words = log2 N * level * 2 * N);
+ * level must be even, 1 <= base_log <= 28, base_log * level <= 64.  Converted
+ * on the device like the BSK.  Errors: INVALID_ARG, UNSUPPORTED_PARAMS, CUDA,
+ * OOM. */
+int rosetta_upload_trace_keys(rosetta_ctx *ctx, const uint64_t *keys, size_t n_words, uint32_t base_log,
+                              uint32_t level, int src_is_device, void *stream);
+
+/* RLWE trace of `batch` GLWE ciphertexts glwe_in [batch][2][N] into glwe_out
+ * (same layout, device memory, no overlap): for each step
+ *     c <- c + (0, B') - sum_lev D_lev(A') * key_s[lev],  (A', B') = c(X^k)
+ * with D the signed gadget digits (base_log, level).  The output encrypts N
+ * times the input's constant coefficient (zeros elsewhere): N has no inverse
+ * mod 2^64, so callers encode the message at Delta / N.  Exact words (same
+ * products mod 2^64 as the definition).  Errors: INVALID_ARG, KEYS_MISSING,
+ * CUDA. */
+int rosetta_trace_batch(rosetta_ctx *ctx, const uint64_t *glwe_in, uint32_t batch, uint64_t *glwe_out,
+                        void *stream);
+
 /* Same computation and result as rosetta_pbs_batch, for callers that cannot
  * allocate device memory during the call (their device memory belongs to
  * another allocator, or their serving loop forbids allocation after

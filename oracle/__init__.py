@@ -79,6 +79,10 @@ def lib():
             L.orc_blind_rotate.argtypes = [P, pp, P, P, P]
             L.orc_sample_extract.argtypes = [P, P, u32, u32]
             L.orc_blind_rotate_glwe.argtypes = [P, pp, P, P, P]
+            L.orc_automorphism.argtypes = [P, P, u32, u32]
+            L.orc_auto_key_gen.argtypes = [P, P, u32, u32, u32, u32, P, P]
+            L.orc_trace_step.argtypes = [P, P, u32, u32, u32, u32]
+            L.orc_trace.argtypes = [P, P, u32, u32, u32]
             L.orc_keyswitch.argtypes = [P, pp, P, P]
             L.orc_blind_rotate_extract.argtypes = [P, pp, P, P, P]
             L.orc_pbs.argtypes = [P, pp, P, P, P, P]
@@ -300,6 +304,47 @@ def blind_rotate_glwe_batch(p, bsk, lwe, glwe_in, threads=None) -> np.ndarray:
 
     with ThreadPoolExecutor(threads or default_threads()) as ex:
         list(ex.map(one, range(lwe.shape[0])))
+    return out
+
+
+# ---------------------------------------------------------------- RLWE trace (k = 1)
+
+def automorphism(a, k: int) -> np.ndarray:
+    a = _c(a)
+    out = np.empty_like(a)
+    lib().orc_automorphism(_u64p(out), _u64p(a), k, a.size)
+    return out
+
+
+def trace_exponents(N: int) -> list:
+    """Automorphism exponents of the trace steps, in order: N+1, N/2+1, ..., 3."""
+    logN = N.bit_length() - 1
+    return [(1 << (logN - s)) + 1 for s in range(logN)]
+
+
+def trace_keys(S, base_log: int, level: int, mask, noise) -> np.ndarray:
+    """[log2 N][level][2][N] automorphism keys; mask/noise [log2 N][level][N]."""
+    S = _c(S).reshape(-1)
+    N = S.size
+    ks = trace_exponents(N)
+    out = np.empty((len(ks), level, 2, N), np.uint64)
+    mask, noise = _c(mask), _c(noise)
+    for s, k in enumerate(ks):
+        lib().orc_auto_key_gen(_u64p(out[s]), _u64p(S), N, k, base_log, level, _u64p(mask[s]), _u64p(noise[s]))
+    return out
+
+
+def trace_batch(keys, glwe, base_log: int, level: int, threads=None) -> np.ndarray:
+    """[batch][2][N] traces of GLWE ciphertexts (k = 1)."""
+    keys = _c(keys)
+    out = _c(glwe).copy()
+    N = out.shape[-1]
+
+    def one(b):
+        lib().orc_trace(_u64p(out[b]), _u64p(keys), N, base_log, level)
+
+    with ThreadPoolExecutor(threads or default_threads()) as ex:
+        list(ex.map(one, range(out.shape[0])))
     return out
 
 

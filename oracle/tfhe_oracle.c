@@ -321,6 +321,84 @@ void orc_keyswitch(uint64_t *out, const orc_params *P, const uint64_t *ksk, cons
   }
 }
 
+/* ------------------------------------------------------------------------ */
+/* RLWE trace (Background, "Scheme Conversion and Other Primitives", RLWE    */
+/* Trace Computation: a logarithmic sequence of Galois automorphisms and     */
+/* additions leaves only the constant term).  k = 1.                          */
+/* ------------------------------------------------------------------------ */
+
+/* out = a(X^k) in R_{N,q} for odd k: coefficient t moves to t k mod 2N, with
+ * a sign flip when that exponent lies in [N, 2N).  out must not alias a. */
+void orc_automorphism(uint64_t *out, const uint64_t *a, uint32_t k, uint32_t N) {
+  for (uint32_t t = 0; t < N; ++t) {
+    uint64_t e = ((uint64_t)t * k) % (2 * (uint64_t)N);
+    if (e < N) out[e] = a[t];
+    else out[e - N] = (uint64_t)0 - a[t];
+  }
+}
+
+/* Automorphism key for X -> X^k: row l (l = 1..level) is a GLWE encryption
+ * under S of sigma_k(S) * 2^(64 - l*base_log).  Layout [level][2][N].
+ * mask: [level][N], noise: [level][N]. */
+void orc_auto_key_gen(uint64_t *key, const uint64_t *S, uint32_t N, uint32_t k, uint32_t base_log,
+                      uint32_t level, const uint64_t *mask, const uint64_t *noise) {
+  uint64_t *sig = (uint64_t *)malloc(sizeof(uint64_t) * N);
+  uint64_t *msg = (uint64_t *)malloc(sizeof(uint64_t) * N);
+  orc_automorphism(sig, S, k, N);
+  for (uint32_t l = 1; l <= level; ++l) {
+    for (uint32_t t = 0; t < N; ++t) msg[t] = sig[t] << (64 - l * base_log);
+    orc_glwe_encrypt(key + (size_t)(l - 1) * 2 * N, S, 1, N, msg, mask + (size_t)(l - 1) * N,
+                     noise + (size_t)(l - 1) * N);
+  }
+  free(sig);
+  free(msg);
+}
+
+/* c <- c + KS(sigma_k(c)) with KS(A', B') = (0, B') - sum_l D_l(A') * key[l]:
+ * the automorphed ciphertext is an encryption under sigma_k(S); the key
+ * switch brings it back under S, and the sum doubles the coefficients the
+ * automorphism fixes and cancels the ones it negates. */
+void orc_trace_step(uint64_t *c, const uint64_t *key, uint32_t N, uint32_t k, uint32_t base_log, uint32_t level) {
+  uint64_t *sA = (uint64_t *)malloc(sizeof(uint64_t) * N);
+  uint64_t *sB = (uint64_t *)malloc(sizeof(uint64_t) * N);
+  uint64_t *dig = (uint64_t *)malloc(sizeof(uint64_t) * N);
+  uint64_t *prod = (uint64_t *)calloc(2 * (size_t)N, sizeof(uint64_t));
+  int64_t d[64];
+  orc_automorphism(sA, c, k, N);
+  orc_automorphism(sB, c + N, k, N);
+  for (uint32_t l = 1; l <= level; ++l) {
+    for (uint32_t t = 0; t < N; ++t) {
+      orc_decompose(sA[t], base_log, level, d);
+      dig[t] = (uint64_t)d[l - 1];
+    }
+    for (uint32_t comp = 0; comp < 2; ++comp)
+      orc_poly_mul_acc(prod + (size_t)comp * N, dig, key + ((size_t)(l - 1) * 2 + comp) * N, N);
+  }
+  for (uint32_t t = 0; t < N; ++t) {
+    c[t] -= prod[t];
+    c[N + t] += sB[t] - prod[N + t];
+  }
+  free(sA);
+  free(sB);
+  free(dig);
+  free(prod);
+}
+
+/* Trace to the constant coefficient: for j = log2 N down to 1, apply the
+ * step with k = 2^j + 1 (key j-1 of keys [log2 N][level][2][N]: keys[0] for
+ * k = N + 1, ..., keys[log2 N - 1] for k = 3).  The phase becomes N times the
+ * constant coefficient of the input phase, zeros elsewhere; on the torus
+ * Z_{2^64} N has no inverse, so the factor N stays (the caller encodes the
+ * message at scale Delta / N). */
+void orc_trace(uint64_t *c, const uint64_t *keys, uint32_t N, uint32_t base_log, uint32_t level) {
+  uint32_t logN = 0;
+  while ((1u << logN) < N) ++logN;
+  for (uint32_t s = 0; s < logN; ++s) {
+    uint32_t k = (1u << (logN - s)) + 1;
+    orc_trace_step(c, keys + (size_t)s * level * 2 * N, N, k, base_log, level);
+  }
+}
+
 void orc_blind_rotate_extract(uint64_t *lwe_big, const orc_params *P, const uint64_t *bsk,
                               const uint64_t *lwe, const uint64_t *lut) {
   uint64_t *acc = (uint64_t *)malloc(sizeof(uint64_t) * (size_t)(P->k + 1) * P->N);

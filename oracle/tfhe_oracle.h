@@ -79,6 +79,13 @@ void orc_pbs(uint64_t *out, const orc_params *P, const uint64_t *bsk, const uint
              const uint64_t *lwe, const uint64_t *lut);
 uint64_t orc_decrypt(const uint64_t *ct, const uint64_t *s, uint32_t n, uint32_t msg_bits);
 
+/* RLWE trace (k = 1) */
+void orc_automorphism(uint64_t *out, const uint64_t *a, uint32_t k, uint32_t N);
+void orc_auto_key_gen(uint64_t *key, const uint64_t *S, uint32_t N, uint32_t k, uint32_t base_log,
+                      uint32_t level, const uint64_t *mask, const uint64_t *noise);
+void orc_trace_step(uint64_t *c, const uint64_t *key, uint32_t N, uint32_t k, uint32_t base_log, uint32_t level);
+void orc_trace(uint64_t *c, const uint64_t *keys, uint32_t N, uint32_t base_log, uint32_t level);
+
 #ifdef __cplusplus
 }
 #endif

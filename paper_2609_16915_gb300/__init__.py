@@ -22,7 +22,8 @@ STATUS = {0: "ok", -1: "invalid argument", -2: "unsupported parameters", -3: "ke
 
 EXPORTS = ("rosetta_params_init", "rosetta_upload_bsk", "rosetta_upload_ksk", "rosetta_pbs_batch",
            "rosetta_blind_rotate_extract_batch", "rosetta_keyswitch_batch", "rosetta_pbs_batch_multi_lut",
-           "rosetta_blind_rotate_glwe_batch", "rosetta_pbs_batch_noalloc",
+           "rosetta_blind_rotate_glwe_batch", "rosetta_upload_trace_keys", "rosetta_trace_batch",
+           "rosetta_pbs_batch_noalloc",
            "rosetta_sync_status", "rosetta_destroy", "rosetta_status_string")
 
 
@@ -59,6 +60,8 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     L.rosetta_pbs_batch_noalloc.argtypes = [vp, u64p, u32, u64p, u64p, vp]
     L.rosetta_pbs_batch_multi_lut.argtypes = [vp, u64p, u32, u64p, u32, vp, u64p, vp]
     L.rosetta_blind_rotate_glwe_batch.argtypes = [vp, u64p, u32, u64p, u64p, vp]
+    L.rosetta_upload_trace_keys.argtypes = [vp, u64p, ctypes.c_size_t, u32, u32, ctypes.c_int, vp]
+    L.rosetta_trace_batch.argtypes = [vp, u64p, u32, u64p, vp]
     L.rosetta_sync_status.argtypes = [vp, vp]
     L.rosetta_destroy.argtypes = [vp]
     L.rosetta_destroy.restype = None
@@ -177,6 +180,18 @@ class Context:
                                                       _stream(stream)))
         return glwe_out
 
+    def rosetta_upload_trace_keys(self, keys, base_log, level, stream=None):
+        n = keys.numel() if hasattr(keys, "numel") else keys.size
+        _check("rosetta_upload_trace_keys",
+               load().rosetta_upload_trace_keys(self._h, _ptr(keys), n, base_log, level, int(_is_device(keys)),
+                                                _stream(stream)))
+
+    def rosetta_trace_batch(self, glwe_in, glwe_out, stream=None):
+        """RLWE trace of glwe_in [batch][2][N] (device) into glwe_out."""
+        _check("rosetta_trace_batch", load().rosetta_trace_batch(self._h, _ptr(glwe_in), glwe_in.shape[0],
+                                                                 _ptr(glwe_out), _stream(stream)))
+        return glwe_out
+
     def rosetta_pbs_batch_noalloc(self, lwe_in, lut, lwe_out, stream=None):
         """rosetta_pbs_batch without any device allocation in the call (fixed
         in-library scratch; device buffers only, bounded batch)."""
@@ -196,4 +211,6 @@ class Context:
     keyswitch_batch = rosetta_keyswitch_batch
     pbs_batch_multi_lut = rosetta_pbs_batch_multi_lut
     blind_rotate_glwe_batch = rosetta_blind_rotate_glwe_batch
+    upload_trace_keys = rosetta_upload_trace_keys
+    trace_batch = rosetta_trace_batch
     sync_status = rosetta_sync_status

@@ -7,7 +7,8 @@
 // products returns the plain product).
 //
 // Output layout [i][prime][row][component][N] uint32, so that one CTA of the
-// blind-rotation kernel streams one contiguous block per CMux step.
+// blind-rotation (or trace) kernel streams one contiguous block per step.
+// The same conversion serves the trace's automorphism keys.
 #include "internal.h"
 #include "ntt.cuh"
 
@@ -55,30 +56,35 @@ __global__ void __launch_bounds__((1 << LOGN) / 8)
 }
 
 template <int LOGN>
-static cudaError_t launch_bsk_t(const uint64_t *raw, uint32_t *out, const uint2 *tw, const CrtConsts &cc, uint32_t n,
-                                uint32_t level, cudaStream_t s) {
+static cudaError_t launch_key_t(const uint64_t *raw, uint32_t *out, const uint2 *tw, const CrtConsts &cc,
+                                uint32_t count, uint32_t rows, cudaStream_t s) {
   using S = NttShape<LOGN, 8>;
   const size_t smem = S::N * sizeof(uint2) + S::XB_WORDS * sizeof(uint32_t);
   auto kern = bsk_transform_kernel<LOGN>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  const uint32_t rows = 2 * level;
-  dim3 grid(n * rows * 2, kPrimes, 1);
+  dim3 grid(count * rows * 2, kPrimes, 1);
   kern<<<grid, S::T, smem, s>>>(raw, out, tw, cc, rows);
   return cudaGetLastError();
 }
 
-cudaError_t launch_bsk_transform(const uint64_t *raw, uint32_t *out, const uint2 *tw, const CrtConsts &cc,
-                                 uint32_t logN, uint32_t n, uint32_t level, cudaStream_t s) {
+cudaError_t launch_key_transform(const uint64_t *raw, uint32_t *out, const uint2 *tw, const CrtConsts &cc,
+                                 uint32_t logN, uint32_t count, uint32_t rows, cudaStream_t s) {
   switch (logN) {
-    case 8: return launch_bsk_t<8>(raw, out, tw, cc, n, level, s);
-    case 9: return launch_bsk_t<9>(raw, out, tw, cc, n, level, s);
-    case 10: return launch_bsk_t<10>(raw, out, tw, cc, n, level, s);
-    case 11: return launch_bsk_t<11>(raw, out, tw, cc, n, level, s);
-    case 12: return launch_bsk_t<12>(raw, out, tw, cc, n, level, s);
-    case 13: return launch_bsk_t<13>(raw, out, tw, cc, n, level, s);
+    case 8: return launch_key_t<8>(raw, out, tw, cc, count, rows, s);
+    case 9: return launch_key_t<9>(raw, out, tw, cc, count, rows, s);
+    case 10: return launch_key_t<10>(raw, out, tw, cc, count, rows, s);
+    case 11: return launch_key_t<11>(raw, out, tw, cc, count, rows, s);
+    case 12: return launch_key_t<12>(raw, out, tw, cc, count, rows, s);
+    case 13: return launch_key_t<13>(raw, out, tw, cc, count, rows, s);
     default: return cudaErrorInvalidValue;
   }
+}
+
+// The bootstrapping key: n GGSWs of (k+1) l = 2 l rows each.
+cudaError_t launch_bsk_transform(const uint64_t *raw, uint32_t *out, const uint2 *tw, const CrtConsts &cc,
+                                 uint32_t logN, uint32_t n, uint32_t level, cudaStream_t s) {
+  return launch_key_transform(raw, out, tw, cc, logN, n, 2 * level, s);
 }
 
 }  // namespace rosetta

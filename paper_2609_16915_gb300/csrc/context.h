@@ -28,4 +28,7 @@ struct rosetta_ctx {
   size_t out_words_cap = 0;
   uint64_t *d_lut = nullptr;      // staging for a host LUT  [2^p]
   uint32_t *d_err = nullptr;      // device-side argument error flag (LUT index out of range)
+  uint32_t *d_trk = nullptr;      // trace automorphism keys, transform domain
+  uint32_t trk_base_log = 0, trk_level = 0;
+  bool have_trk = false;
 };

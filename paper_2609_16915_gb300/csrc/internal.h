@@ -53,6 +53,15 @@ struct KsArgs {
   uint32_t batch, kN, n, base_log, level;
 };
 
+struct TraceArgs {
+  const uint64_t *glwe_in;  // [batch][2][N]
+  uint64_t *glwe_out;       // [batch][2][N]
+  const uint32_t *keys;     // transform domain [log2 N][prime][level][2][N]
+  const uint2 *tw;          // [prime][N]
+  uint32_t base_log, level, batch;
+  CrtConsts cc;
+};
+
 // host-side tables (tables.cu)
 bool build_tables(uint32_t logN, uint2 *tw_host /*[kPrimes][N]*/, CrtConsts *cc);
 
@@ -62,6 +71,11 @@ cudaError_t launch_blind_rotate(const BrArgs &a, uint32_t logN, bool dig16, cuda
 cudaError_t launch_bsk_transform(const uint64_t *raw, uint32_t *out, const uint2 *tw, const CrtConsts &cc,
                                  uint32_t logN, uint32_t n, uint32_t level, cudaStream_t s);
 cudaError_t launch_keyswitch(const KsArgs &a, cudaStream_t s);
+// transform `count` raw keys [count][rows][2][N] to [count][prime][rows][2][N]
+cudaError_t launch_key_transform(const uint64_t *raw, uint32_t *out, const uint2 *tw, const CrtConsts &cc,
+                                 uint32_t logN, uint32_t count, uint32_t rows, cudaStream_t s);
+size_t trace_smem_bytes(uint32_t logN, uint32_t level);
+cudaError_t launch_trace(const TraceArgs &a, uint32_t logN, cudaStream_t s);
 cudaError_t launch_ksk_corr(const uint64_t *ksk, uint64_t *corr, uint32_t rows, uint32_t n, uint32_t base_log,
                             cudaStream_t s);
 

@@ -413,6 +413,84 @@ int rosetta_blind_rotate_glwe_batch(rosetta_ctx *c, const uint64_t *lwe_in, uint
   return e == cudaSuccess ? ROSETTA_OK : cuda_fail(e);
 }
 
+int rosetta_upload_trace_keys(rosetta_ctx *c, const uint64_t *keys, size_t n_words, uint32_t base_log,
+                              uint32_t level, int src_is_device, void *stream) {
+  if (!c || !keys) return ROSETTA_ERR_INVALID_ARG;
+  const rosetta_params &p = c->prm;
+  if (base_log < 1 || base_log > 28 || level < 2 || (level & 1u) || base_log * level > 64)
+    return ROSETTA_ERR_UNSUPPORTED_PARAMS;
+  if (c->logN > 12) return ROSETTA_ERR_UNSUPPORTED_PARAMS;
+  // exact CRT: level N 2^(base_log-1) 2^63 below M/2 > 2^114
+  {
+    int e = 0;
+    while ((1ull << e) < (uint64_t)level * p.poly_size) ++e;
+    if (63 + (base_log - 1) + e + 1 > 115) return ROSETTA_ERR_UNSUPPORTED_PARAMS;
+  }
+  int max_smem = 0;
+  cudaDeviceGetAttribute(&max_smem, cudaDevAttrMaxSharedMemoryPerBlockOptin, c->device);
+  if (trace_smem_bytes(c->logN, level) > (size_t)max_smem) return ROSETTA_ERR_UNSUPPORTED_PARAMS;
+  const size_t want = (size_t)c->logN * level * 2 * p.poly_size;
+  if (n_words != want || !aligned8(keys)) return ROSETTA_ERR_INVALID_ARG;
+  if (cudaSetDevice(c->device) != cudaSuccess) return ROSETTA_ERR_CUDA;
+  cudaStream_t s = as_stream(stream);
+  const uint64_t *src = keys;
+  uint64_t *tmp = nullptr;
+  cudaError_t e = cudaSuccess;
+  if (!src_is_device) {
+    e = cudaMallocAsync(reinterpret_cast<void **>(&tmp), want * 8, s);
+    if (e != cudaSuccess) return cuda_fail(e);
+    e = cudaMemcpyAsync(tmp, keys, want * 8, cudaMemcpyHostToDevice, s);
+    if (e != cudaSuccess) {
+      cudaFreeAsync(tmp, s);
+      return cuda_fail(e);
+    }
+    src = tmp;
+  }
+  if (c->d_trk && c->trk_level != level) {
+    cudaFree(c->d_trk);
+    c->d_trk = nullptr;
+  }
+  if (!c->d_trk) e = cudaMalloc(&c->d_trk, want * kPrimes * sizeof(uint32_t));
+  if (e != cudaSuccess) {
+    if (tmp) cudaFreeAsync(tmp, s);
+    return cuda_fail(e);
+  }
+  e = launch_key_transform(src, c->d_trk, c->d_tw, c->cc, c->logN, c->logN, level, s);
+  if (tmp) cudaFreeAsync(tmp, s);
+  if (e != cudaSuccess) return cuda_fail(e);
+  if (!src_is_device) {
+    e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail(e);
+  }
+  c->trk_base_log = base_log;
+  c->trk_level = level;
+  c->have_trk = true;
+  return ROSETTA_OK;
+}
+
+int rosetta_trace_batch(rosetta_ctx *c, const uint64_t *glwe_in, uint32_t batch, uint64_t *glwe_out, void *stream) {
+  if (!c) return ROSETTA_ERR_INVALID_ARG;
+  if (batch == 0) return ROSETTA_OK;
+  if (!glwe_in || !glwe_out) return ROSETTA_ERR_INVALID_ARG;
+  if (!c->have_trk) return ROSETTA_ERR_KEYS_MISSING;
+  if (cudaSetDevice(c->device) != cudaSuccess) return ROSETTA_ERR_CUDA;
+  const size_t gbytes = (size_t)batch * 2 * c->prm.poly_size * 8;
+  if (!is_device_ptr(glwe_in) || !is_device_ptr(glwe_out) || !aligned8(glwe_in) || !aligned8(glwe_out) ||
+      overlaps(glwe_in, gbytes, glwe_out, gbytes))
+    return ROSETTA_ERR_INVALID_ARG;
+  TraceArgs a{};
+  a.glwe_in = glwe_in;
+  a.glwe_out = glwe_out;
+  a.keys = c->d_trk;
+  a.tw = c->d_tw;
+  a.base_log = c->trk_base_log;
+  a.level = c->trk_level;
+  a.batch = batch;
+  a.cc = c->cc;
+  cudaError_t e = launch_trace(a, c->logN, as_stream(stream));
+  return e == cudaSuccess ? ROSETTA_OK : cuda_fail(e);
+}
+
 int rosetta_sync_status(rosetta_ctx *c, void *stream) {
   if (!c) return ROSETTA_ERR_INVALID_ARG;
   if (cudaSetDevice(c->device) != cudaSuccess) return ROSETTA_ERR_CUDA;
@@ -440,6 +518,7 @@ void rosetta_destroy(rosetta_ctx *c) {
   cudaFree(c->d_out);
   cudaFree(c->d_lut);
   cudaFree(c->d_err);
+  cudaFree(c->d_trk);
   delete c;
 }
 

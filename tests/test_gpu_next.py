@@ -109,3 +109,69 @@ def test_glwe_blind_rotation_rejects_host_buffers():
     with pytest.raises(R.RosettaError) as e:
         ctx.blind_rotate_glwe_batch(lwe, glwe, np.zeros_like(glwe))
     assert e.value.status == -1
+
+
+# ------------------------------------------------------------------ RLWE trace
+
+def _trace_keys(p, base_log, level, noiseless, seed):
+    g = np.random.default_rng(seed)
+    S = g.integers(0, 2, size=p.N, dtype=np.uint64)
+    steps = p.N.bit_length() - 1
+    mask = g.integers(0, 2**64, size=(steps, level, p.N), dtype=np.uint64, endpoint=False)
+    noise = np.rint(g.standard_normal((steps, level, p.N)) * 2.0 ** 13).astype(np.int64).view(np.uint64)
+    if noiseless:
+        mask[:] = 0
+        noise[:] = 0
+    return S, O.trace_keys(S, base_log, level, mask, noise)
+
+
+@pytest.mark.parametrize("name,base_log,level", [("tiny", 16, 4), ("standard", 12, 4), ("gpt2_mlp", 16, 2)])
+def test_trace_bitexact(name, base_log, level):
+    """GPU trace word for word against the oracle (random keys and inputs)."""
+    p = W.CONFIGS[name]
+    S, keys = _trace_keys(p, base_log, level, False, 3)
+    glwe = W.uniform_u64((5, 2, p.N), W.rng(p.seed, "sample", 41))
+    import paper_2609_16915_gb300 as R
+    ctx = R.Context(p)
+    ctx.upload_trace_keys(G.to_dev(keys), base_log, level)
+    out = G.empty_dev(5, 2, p.N)
+    ctx.trace_batch(G.to_dev(glwe), out)
+    ctx.sync_status()
+    assert np.array_equal(G.to_host(out), O.trace_batch(keys, glwe, base_log, level))
+
+
+def test_trace_noiseless_closed_form_on_gpu():
+    """Noiseless keys, gadget over all 64 bits: phase(out) = (N phase(in)[0], 0, ..)."""
+    p = W.CONFIGS["standard"]
+    S, keys = _trace_keys(p, 16, 4, True, 4)
+    glwe = W.uniform_u64((3, 2, p.N), W.rng(p.seed, "sample", 42))
+    import paper_2609_16915_gb300 as R
+    ctx = R.Context(p)
+    ctx.upload_trace_keys(G.to_dev(keys), 16, 4)
+    out = G.empty_dev(3, 2, p.N)
+    ctx.trace_batch(G.to_dev(glwe), out)
+    ctx.sync_status()
+    got = G.to_host(out)
+    for b in range(3):
+        ph_in = O.glwe_phase(S.reshape(1, -1), glwe[b])
+        ph = O.glwe_phase(S.reshape(1, -1), got[b])
+        assert int(ph[0]) == (p.N * int(ph_in[0])) % (1 << 64)
+        assert not ph[1:].any()
+
+
+def test_trace_argument_checks():
+    import paper_2609_16915_gb300 as R
+    p = W.CONFIGS["standard"]
+    ctx = R.Context(p)
+    glwe = G.to_dev(np.zeros((1, 2, p.N), np.uint64))
+    with pytest.raises(R.RosettaError) as e:
+        ctx.trace_batch(glwe, G.empty_dev(1, 2, p.N))
+    assert e.value.status == -3                     # keys missing
+    keys = np.zeros((11, 3, 2, p.N), np.uint64)
+    with pytest.raises(R.RosettaError) as e:
+        ctx.upload_trace_keys(G.to_dev(keys), 16, 3)   # odd level
+    assert e.value.status == -2
+    big = R.Context(W.CONFIGS["llama_silu"])
+    with pytest.raises(R.RosettaError) as e:
+        big.upload_trace_keys(G.to_dev(np.zeros((13, 2, 2, 8192), np.uint64)), 16, 2)
+    assert e.value.status == -2                     # N = 8192 not supported for the trace

@@ -372,3 +372,69 @@ def test_glwe_blind_rotation_decrypts_to_rotated_table():
     for b in range(8):
         ph = int(O.glwe_phase(keys.glwe_key, out[b])[0])
         assert ((ph + (1 << (sh - 1))) >> sh) % (1 << (p.msg_bits + 1)) == W.lut_codes(p)[codes[b]]
+
+
+# ------------------------------------------------------------------ RLWE trace
+
+@pytest.mark.parametrize("N", [8, 64])
+def test_automorphism_is_a_ring_homomorphism(N):
+    rs = random.Random(N + 1)
+    a, b = rnd_u64(rs, N), rnd_u64(rs, N)
+    for k in [1, 3, 5, N + 1, 2 * N - 1]:
+        assert np.array_equal(O.automorphism(O.poly_mul(a, b), k), O.poly_mul(O.automorphism(a, k), O.automorphism(b, k)))
+        for k2 in [3, N - 1]:
+            assert np.array_equal(O.automorphism(O.automorphism(a, k), k2), O.automorphism(a, (k * k2) % (2 * N)))
+    assert np.array_equal(O.automorphism(a, 1), a)
+    # X -> X^(N+1) = -X negates the odd coefficients
+    sign = np.array([1 if t % 2 == 0 else -1 for t in range(N)], dtype=object)
+    assert [int(x) for x in O.automorphism(a, N + 1)] == [int(x) * int(s) % Q for x, s in zip(a, sign)]
+
+
+def _trace_setup(N, base_log, level, noiseless, seed):
+    rs = np.random.default_rng(seed)
+    S = (rs.integers(0, 2, size=N, dtype=np.uint64)).astype(np.uint64)
+    steps = N.bit_length() - 1
+    mask = rs.integers(0, 2**64, size=(steps, level, N), dtype=np.uint64, endpoint=False)
+    noise = np.rint(rs.standard_normal((steps, level, N)) * 2.0 ** 13).astype(np.int64).view(np.uint64)
+    if noiseless:
+        mask[:] = 0
+        noise[:] = 0
+    return S, O.trace_keys(S, base_log, level, mask, noise)
+
+
+@pytest.mark.parametrize("N", [16, 256])
+def test_trace_noiseless_exact_gadget_closed_form(N):
+    """Noiseless automorphism keys with a gadget covering all 64 bits (no
+    rounding): the trace's phase is exactly N * phase[0] at coefficient 0
+    and 0 elsewhere."""
+    S, keys = _trace_setup(N, 16, 4, True, N)
+    rs = random.Random(N + 7)
+    c = rnd_u64(rs, 2 * N).reshape(1, 2, N)
+    out = O.trace_batch(keys, c, 16, 4)
+    ph_in = O.glwe_phase(S.reshape(1, N), c[0])
+    ph_out = O.glwe_phase(S.reshape(1, N), out[0])
+    assert int(ph_out[0]) == (N * int(ph_in[0])) % Q
+    assert not ph_out[1:].any()
+
+
+def test_trace_real_keys_isolates_constant_term():
+    """Real (masked, noisy) keys: phase(Tr(c)) = N * phase(c)[0] at
+    coefficient 0 and ~0 elsewhere, within the accumulated rounding and key
+    noise of log2 N key switches."""
+    N, bl, lv = 256, 8, 4
+    S, keys = _trace_setup(N, bl, lv, False, 5)
+    rs = np.random.default_rng(9)
+    msg = (rs.integers(0, 16, size=N, dtype=np.uint64) << np.uint64(52)).astype(np.uint64)
+    c = O.glwe_encrypt(S.reshape(1, N), msg, rs.integers(0, 2**64, size=(1, N), dtype=np.uint64, endpoint=False),
+                       np.zeros(N, np.uint64)).reshape(1, 2, N)
+    out = O.trace_batch(keys, c, bl, lv)
+    ph = O.glwe_phase(S.reshape(1, N), out[0]).astype(object)
+    want = [(N * int(msg[0])) % Q] + [0] * (N - 1)
+    err = [((int(a) - b + Q // 2) % Q) - Q // 2 for a, b in zip(ph, want)]
+    # per step: decomposition rounding (< 2^(63 - bl*lv) per coefficient times |S| <= N)
+    # plus key noise (|d| <= 2^(bl-1), N lv terms of 6 sigma); the trace doubles what came before
+    steps = N.bit_length() - 1
+    per_step = N * (1 << (63 - bl * lv)) + N * lv * (1 << (bl - 1)) * 6 * (1 << 13)
+    bound = per_step * (2 ** steps)
+    assert max(abs(e) for e in err) < bound
+    assert bound < (1 << 52) * N // 2     # the bound itself leaves the message readable

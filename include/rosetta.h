@@ -181,6 +181,19 @@ int rosetta_upload_trace_keys(rosetta_ctx *ctx, const uint64_t *keys, size_t n_w
 int rosetta_trace_batch(rosetta_ctx *ctx, const uint64_t *glwe_in, uint32_t batch, uint64_t *glwe_out,
                         void *stream);
 
+/* Plaintext x ciphertext polynomial product (k = 1, N <= 4096), the linear
+ * mapping of the lookup protocol (Cryptographic Lookup Protocol, Steps 2 and
+ * 3: [[t]] = p(X) [[x]] + q(X), [[r_s]] = a_s(X) [[x]] + b_s(X), with the
+ * real coefficients encoded as integers by the caller):
+ *   glwe_out[b] = (P * A_b, P * B_b + Q)   in Z_{2^64}[X]/(X^N+1)
+ *   glwe_in, glwe_out [batch][2][N] uint64, device memory, no overlap
+ *   plain_mul [N] int64 P, HOST memory (any value; products are mod 2^64)
+ *   plain_add [N] uint64 Q (host or device) or NULL for Q = 0
+ * Exact words.  Returns after the work completes.  Errors: INVALID_ARG,
+ * UNSUPPORTED_PARAMS, CUDA, OOM. */
+int rosetta_plaintext_mul_batch(rosetta_ctx *ctx, const uint64_t *glwe_in, uint32_t batch, const int64_t *plain_mul,
+                                const uint64_t *plain_add, uint64_t *glwe_out, void *stream);
+
 /* Same computation and result as rosetta_pbs_batch, for callers that cannot
  * allocate device memory during the call (their device memory belongs to
  * another allocator, or their serving loop forbids allocation after

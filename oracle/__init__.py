@@ -83,6 +83,7 @@ def lib():
             L.orc_auto_key_gen.argtypes = [P, P, u32, u32, u32, u32, P, P]
             L.orc_trace_step.argtypes = [P, P, u32, u32, u32, u32]
             L.orc_trace.argtypes = [P, P, u32, u32, u32]
+            L.orc_plaintext_mul.argtypes = [P, P, P, P, u32]
             L.orc_keyswitch.argtypes = [P, pp, P, P]
             L.orc_blind_rotate_extract.argtypes = [P, pp, P, P, P]
             L.orc_pbs.argtypes = [P, pp, P, P, P, P]
@@ -345,6 +346,18 @@ def trace_batch(keys, glwe, base_log: int, level: int, threads=None) -> np.ndarr
 
     with ThreadPoolExecutor(threads or default_threads()) as ex:
         list(ex.map(one, range(out.shape[0])))
+    return out
+
+
+def plaintext_mul_batch(glwe, plain_mul, plain_add=None) -> np.ndarray:
+    """[batch][2][N]: (P * A, P * B + Q) for each GLWE; P given as signed ints."""
+    glwe = _c(glwe)
+    P = np.asarray(plain_mul, dtype=np.int64).view(np.uint64).copy()
+    Qp = _c(plain_add) if plain_add is not None else None
+    out = np.empty_like(glwe)
+    N = glwe.shape[-1]
+    for b in range(glwe.shape[0]):
+        lib().orc_plaintext_mul(_u64p(out[b]), _u64p(glwe[b]), _u64p(P), _u64p(Qp) if Qp is not None else None, N)
     return out
 
 

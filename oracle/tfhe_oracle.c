@@ -399,6 +399,15 @@ void orc_trace(uint64_t *c, const uint64_t *keys, uint32_t N, uint32_t base_log,
   }
 }
 
+/* Plaintext x ciphertext product (k = 1): (P * A, P * B + Q), the linear
+ * mapping of the lookup protocol.  Q may be NULL. */
+void orc_plaintext_mul(uint64_t *out, const uint64_t *c, const uint64_t *P, const uint64_t *Qp, uint32_t N) {
+  orc_poly_mul(out, P, c, N);
+  orc_poly_mul(out + N, P, c + N, N);
+  if (Qp)
+    for (uint32_t t = 0; t < N; ++t) out[N + t] += Qp[t];
+}
+
 void orc_blind_rotate_extract(uint64_t *lwe_big, const orc_params *P, const uint64_t *bsk,
                               const uint64_t *lwe, const uint64_t *lut) {
   uint64_t *acc = (uint64_t *)malloc(sizeof(uint64_t) * (size_t)(P->k + 1) * P->N);

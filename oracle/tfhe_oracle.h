@@ -85,6 +85,7 @@ void orc_auto_key_gen(uint64_t *key, const uint64_t *S, uint32_t N, uint32_t k, 
                       uint32_t level, const uint64_t *mask, const uint64_t *noise);
 void orc_trace_step(uint64_t *c, const uint64_t *key, uint32_t N, uint32_t k, uint32_t base_log, uint32_t level);
 void orc_trace(uint64_t *c, const uint64_t *keys, uint32_t N, uint32_t base_log, uint32_t level);
+void orc_plaintext_mul(uint64_t *out, const uint64_t *c, const uint64_t *P, const uint64_t *Qp, uint32_t N);
 
 #ifdef __cplusplus
 }

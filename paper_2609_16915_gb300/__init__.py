@@ -23,6 +23,7 @@ STATUS = {0: "ok", -1: "invalid argument", -2: "unsupported parameters", -3: "ke
 EXPORTS = ("rosetta_params_init", "rosetta_upload_bsk", "rosetta_upload_ksk", "rosetta_pbs_batch",
            "rosetta_blind_rotate_extract_batch", "rosetta_keyswitch_batch", "rosetta_pbs_batch_multi_lut",
            "rosetta_blind_rotate_glwe_batch", "rosetta_upload_trace_keys", "rosetta_trace_batch",
+           "rosetta_plaintext_mul_batch",
            "rosetta_pbs_batch_noalloc",
            "rosetta_sync_status", "rosetta_destroy", "rosetta_status_string")
 
@@ -62,6 +63,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     L.rosetta_blind_rotate_glwe_batch.argtypes = [vp, u64p, u32, u64p, u64p, vp]
     L.rosetta_upload_trace_keys.argtypes = [vp, u64p, ctypes.c_size_t, u32, u32, ctypes.c_int, vp]
     L.rosetta_trace_batch.argtypes = [vp, u64p, u32, u64p, vp]
+    L.rosetta_plaintext_mul_batch.argtypes = [vp, u64p, u32, u64p, u64p, u64p, vp]
     L.rosetta_sync_status.argtypes = [vp, vp]
     L.rosetta_destroy.argtypes = [vp]
     L.rosetta_destroy.restype = None
@@ -192,6 +194,18 @@ class Context:
                                                                  _ptr(glwe_out), _stream(stream)))
         return glwe_out
 
+    def rosetta_plaintext_mul_batch(self, glwe_in, plain_mul, glwe_out, plain_add=None, stream=None):
+        """(P * A, P * B + Q) for glwe_in [batch][2][N] (device); plain_mul: host int64 [N]."""
+        n = glwe_in.shape[-1]
+        for name, v in (("plain_mul", plain_mul), ("plain_add", plain_add)):
+            if v is not None and (v.shape != (n,) or v.dtype.itemsize != 8):
+                raise ValueError(f"{name} must hold {n} 64-bit words")
+        _check("rosetta_plaintext_mul_batch",
+               load().rosetta_plaintext_mul_batch(self._h, _ptr(glwe_in), glwe_in.shape[0], _ptr(plain_mul),
+                                                  None if plain_add is None else _ptr(plain_add), _ptr(glwe_out),
+                                                  _stream(stream)))
+        return glwe_out
+
     def rosetta_pbs_batch_noalloc(self, lwe_in, lut, lwe_out, stream=None):
         """rosetta_pbs_batch without any device allocation in the call (fixed
         in-library scratch; device buffers only, bounded batch)."""
@@ -213,4 +227,5 @@ class Context:
     blind_rotate_glwe_batch = rosetta_blind_rotate_glwe_batch
     upload_trace_keys = rosetta_upload_trace_keys
     trace_batch = rosetta_trace_batch
+    plaintext_mul_batch = rosetta_plaintext_mul_batch
     sync_status = rosetta_sync_status

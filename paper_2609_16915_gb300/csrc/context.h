@@ -31,4 +31,7 @@ struct rosetta_ctx {
   uint32_t *d_trk = nullptr;      // trace automorphism keys, transform domain
   uint32_t trk_base_log = 0, trk_level = 0;
   bool have_trk = false;
+  uint64_t *d_pm_raw = nullptr;   // plaintext-multiply gadget rows, raw [8][2][N]
+  uint32_t *d_pm_key = nullptr;   // the same in the transform domain
+  uint64_t *d_pm_add = nullptr;   // staged additive plaintext [N]
 };

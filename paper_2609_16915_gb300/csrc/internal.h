@@ -56,9 +56,10 @@ struct KsArgs {
 struct TraceArgs {
   const uint64_t *glwe_in;  // [batch][2][N]
   uint64_t *glwe_out;       // [batch][2][N]
-  const uint32_t *keys;     // transform domain [log2 N][prime][level][2][N]
+  const uint32_t *keys;     // transform domain [steps][prime][rows][2][N]
+  const uint64_t *plain_add;  // [N] added to the body (plaintext-multiply mode), or null
   const uint2 *tw;          // [prime][N]
-  uint32_t base_log, level, batch;
+  uint32_t base_log, level, batch;  // level = rows of a key (trace); 2 x gadget levels (multiply)
   CrtConsts cc;
 };
 
@@ -76,6 +77,7 @@ cudaError_t launch_key_transform(const uint64_t *raw, uint32_t *out, const uint2
                                  uint32_t logN, uint32_t count, uint32_t rows, cudaStream_t s);
 size_t trace_smem_bytes(uint32_t logN, uint32_t level);
 cudaError_t launch_trace(const TraceArgs &a, uint32_t logN, cudaStream_t s);
+cudaError_t launch_plaintext_mul(const TraceArgs &a, uint32_t logN, cudaStream_t s);
 cudaError_t launch_ksk_corr(const uint64_t *ksk, uint64_t *corr, uint32_t rows, uint32_t n, uint32_t base_log,
                             cudaStream_t s);
 

@@ -491,6 +491,53 @@ int rosetta_trace_batch(rosetta_ctx *c, const uint64_t *glwe_in, uint32_t batch,
   return e == cudaSuccess ? ROSETTA_OK : cuda_fail(e);
 }
 
+int rosetta_plaintext_mul_batch(rosetta_ctx *c, const uint64_t *glwe_in, uint32_t batch, const int64_t *plain_mul,
+                                const uint64_t *plain_add, uint64_t *glwe_out, void *stream) {
+  if (!c) return ROSETTA_ERR_INVALID_ARG;
+  if (batch == 0) return ROSETTA_OK;
+  if (!glwe_in || !plain_mul || !glwe_out) return ROSETTA_ERR_INVALID_ARG;
+  if (c->logN > 12 || c->prm.glwe_dim != 1) return ROSETTA_ERR_UNSUPPORTED_PARAMS;
+  if (cudaSetDevice(c->device) != cudaSuccess) return ROSETTA_ERR_CUDA;
+  const size_t N = c->prm.poly_size;
+  const size_t gbytes = (size_t)batch * 2 * N * 8;
+  if (!is_device_ptr(glwe_in) || !is_device_ptr(glwe_out) || !aligned8(glwe_in) || !aligned8(glwe_out) ||
+      !aligned8(plain_mul) || (plain_add && !aligned8(plain_add)) || overlaps(glwe_in, gbytes, glwe_out, gbytes))
+    return ROSETTA_ERR_INVALID_ARG;
+  if (is_device_ptr(plain_mul)) return ROSETTA_ERR_INVALID_ARG;  // the gadget rows are built on the host
+  // noiseless gadget rows: row c*4 + l of component c is P 2^(64 - (l+1) 16)
+  constexpr uint32_t kBase = 16, kLev = 4, kRows = 2 * kLev;
+  std::vector<uint64_t> raw(kRows * 2 * N, 0);
+  for (uint32_t comp = 0; comp < 2; ++comp)
+    for (uint32_t l = 0; l < kLev; ++l)
+      for (size_t t = 0; t < N; ++t)
+        raw[((comp * kLev + l) * 2 + comp) * N + t] = static_cast<uint64_t>(plain_mul[t]) << (64 - (l + 1) * kBase);
+  cudaStream_t s = as_stream(stream);
+  cudaError_t e = cudaSuccess;
+  if (!c->d_pm_raw) e = cudaMalloc(&c->d_pm_raw, raw.size() * 8);
+  if (e == cudaSuccess && !c->d_pm_key) e = cudaMalloc(&c->d_pm_key, raw.size() * kPrimes * sizeof(uint32_t));
+  if (e == cudaSuccess && !c->d_pm_add) e = cudaMalloc(&c->d_pm_add, N * 8);
+  if (e != cudaSuccess) return cuda_fail(e);
+  e = cudaMemcpyAsync(c->d_pm_raw, raw.data(), raw.size() * 8, cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess && plain_add)
+    e = cudaMemcpyAsync(c->d_pm_add, plain_add, N * 8, cudaMemcpyDefault, s);
+  if (e == cudaSuccess) e = launch_key_transform(c->d_pm_raw, c->d_pm_key, c->d_tw, c->cc, c->logN, 1, kRows, s);
+  if (e != cudaSuccess) return cuda_fail(e);
+  TraceArgs a{};
+  a.glwe_in = glwe_in;
+  a.glwe_out = glwe_out;
+  a.keys = c->d_pm_key;
+  a.plain_add = plain_add ? c->d_pm_add : nullptr;
+  a.tw = c->d_tw;
+  a.base_log = kBase;
+  a.level = kRows;
+  a.batch = batch;
+  a.cc = c->cc;
+  e = launch_plaintext_mul(a, c->logN, s);
+  if (e != cudaSuccess) return cuda_fail(e);
+  e = cudaStreamSynchronize(s);  // the host staging vector goes out of scope
+  return e == cudaSuccess ? ROSETTA_OK : cuda_fail(e);
+}
+
 int rosetta_sync_status(rosetta_ctx *c, void *stream) {
   if (!c) return ROSETTA_ERR_INVALID_ARG;
   if (cudaSetDevice(c->device) != cudaSuccess) return ROSETTA_ERR_CUDA;
@@ -519,6 +566,9 @@ void rosetta_destroy(rosetta_ctx *c) {
   cudaFree(c->d_lut);
   cudaFree(c->d_err);
   cudaFree(c->d_trk);
+  cudaFree(c->d_pm_raw);
+  cudaFree(c->d_pm_key);
+  cudaFree(c->d_pm_add);
   delete c;
 }
 

@@ -21,6 +21,14 @@
 //   2. prime-CTAs transform digit pairs, multiply by key_s, inverse-transform
 //      and send CRT-scaled residues to the owners;
 //   3. owners: A -= X_0, B += sigma_k(B) - X_1.
+//
+// The same kernel in its plaintext-multiply mode computes, in one step,
+// (P * A, P * B + Q) for a plaintext polynomial P (small signed
+// coefficients) and Q: the ciphertext components are split into exact gadget
+// digits (base_log * levels = 64) and multiplied by the rows P 2^(64 - l base_log)
+// of a noiseless "key", which gives P * C exactly; this is the linear mapping
+// a_s(X) [[x]] + b_s(X) of the lookup protocol (Cryptographic Lookup Protocol,
+// Steps 2 and 3).
 #include <cooperative_groups.h>
 
 #include "dsmem.cuh"
@@ -40,7 +48,7 @@ struct TrShape {
   static constexpr int QE = E / 4;
 };
 
-template <int LOGN>
+template <int LOGN, bool PTMUL>
 __global__ void __launch_bounds__(TrShape<LOGN>::T) trace_kernel(const TraceArgs a) {
   using B = TrShape<LOGN>;
   constexpr uint32_t N = B::N, T = B::T, Q = B::Q;
@@ -76,20 +84,24 @@ __global__ void __launch_bounds__(TrShape<LOGN>::T) trace_kernel(const TraceArgs
   cluster.sync();
 
   const uint32_t acc_s = smem_addr(acc), dig_s = smem_addr(dig), res_s = smem_addr(res);
-  const uint32_t bits = a.base_log * a.level;
+  const uint32_t bits = a.base_log * (PTMUL ? a.level / 2 : a.level);
   const uint64_t Bmask = (1ull << a.base_log) - 1;
   const uint64_t Bhalf = 1ull << (a.base_log - 1);
   const uint64_t round_add = bits >= 64 ? 0 : (1ull << (63 - bits));
   const uint32_t round_sh = bits >= 64 ? 0 : 64 - bits;
 
-  for (uint32_t s = 0; s < LOGN; ++s) {
-    const uint32_t k = (1u << (LOGN - s)) + 1u;
+  // multiply mode: level key rows = 2 x gadget levels (component-major)
+  const uint32_t dlev = PTMUL ? a.level / 2 : a.level;
+  constexpr uint32_t STEPS = PTMUL ? 1 : LOGN;
+  for (uint32_t s = 0; s < STEPS; ++s) {
+    const uint32_t k = PTMUL ? 1u : (1u << (LOGN - s)) + 1u;
     uint32_t kinv = k;  // k^{-1} mod 2^32 (Newton), hence mod 2N
 #pragma unroll
     for (int it = 0; it < 5; ++it) kinv *= 2u - k * kinv;
 
     // ---- phase 1: gather sigma_k(c) for the owned quarter ----
-    // coefficient j of a(X^k) is +-a[t] with t = j k^{-1} mod 2N (minus when t >= N)
+    // coefficient j of a(X^k) is +-a[t] with t = j k^{-1} mod 2N (minus when t >= N);
+    // k = 1 in multiply mode (every word is the owner's own)
     uint64_t v[ITEMS];
 #pragma unroll
     for (int m = 0; m < ITEMS; ++m) {
@@ -104,11 +116,12 @@ __global__ void __launch_bounds__(TrShape<LOGN>::T) trace_kernel(const TraceArgs
       const uint32_t c = item / Q, jl = item % Q, j = rank * Q + jl;
       const bool neg = ((j * kinv) & (TWO_N - 1)) >= N;
       const uint64_t w = neg ? 0ull - v[m] : v[m];
-      if (c == 1) {
+      if (!PTMUL && c == 1) {
         sig_b[jl] = w;
       } else {
+        const uint32_t row0 = PTMUL ? c * dlev : 0;
         uint64_t cv = bits >= 64 ? w : (w + round_add) >> round_sh;
-        for (int l = static_cast<int>(a.level) - 1; l >= 0; --l) {
+        for (int l = static_cast<int>(dlev) - 1; l >= 0; --l) {
           const uint64_t d = cv & Bmask;
           cv >>= a.base_log;
           int32_t ds = static_cast<int32_t>(d);
@@ -116,7 +129,7 @@ __global__ void __launch_bounds__(TrShape<LOGN>::T) trace_kernel(const TraceArgs
             ds -= static_cast<int32_t>(Bmask + 1);
             cv += 1;
           }
-          dig[l * Q + jl] = ds;
+          dig[(row0 + l) * Q + jl] = ds;
         }
       }
     }
@@ -185,7 +198,10 @@ __global__ void __launch_bounds__(TrShape<LOGN>::T) trace_kernel(const TraceArgs
       }
       const uint32_t u = (frac + (1u << 27)) >> 28;
       const uint64_t X = sum - static_cast<uint64_t>(u) * a.cc.M_mod64;
-      acc[c * Q + jl] += (c == 1 ? sig_b[jl] : 0ull) - X;
+      if (PTMUL)
+        acc[c * Q + jl] = X + ((c == 1 && a.plain_add) ? a.plain_add[rank * Q + jl] : 0ull);
+      else
+        acc[c * Q + jl] += (c == 1 ? sig_b[jl] : 0ull) - X;
     }
     cluster.sync();
   }
@@ -207,9 +223,9 @@ size_t trace_smem_bytes(uint32_t logN, uint32_t level) {
   return (b + 15) & ~size_t(15);
 }
 
-template <int LOGN>
+template <int LOGN, bool PTMUL>
 static cudaError_t launch_trace_t(const TraceArgs &a, cudaStream_t s) {
-  auto kern = trace_kernel<LOGN>;
+  auto kern = trace_kernel<LOGN, PTMUL>;
   const size_t smem = trace_smem_bytes(LOGN, a.level);
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
@@ -228,15 +244,22 @@ static cudaError_t launch_trace_t(const TraceArgs &a, cudaStream_t s) {
   return cudaLaunchKernelEx(&cfg, kern, a);
 }
 
-cudaError_t launch_trace(const TraceArgs &a, uint32_t logN, cudaStream_t s) {
+template <bool PTMUL>
+static cudaError_t launch_mode(const TraceArgs &a, uint32_t logN, cudaStream_t s) {
   switch (logN) {
-    case 8: return launch_trace_t<8>(a, s);
-    case 9: return launch_trace_t<9>(a, s);
-    case 10: return launch_trace_t<10>(a, s);
-    case 11: return launch_trace_t<11>(a, s);
-    case 12: return launch_trace_t<12>(a, s);
+    case 8: return launch_trace_t<8, PTMUL>(a, s);
+    case 9: return launch_trace_t<9, PTMUL>(a, s);
+    case 10: return launch_trace_t<10, PTMUL>(a, s);
+    case 11: return launch_trace_t<11, PTMUL>(a, s);
+    case 12: return launch_trace_t<12, PTMUL>(a, s);
     default: return cudaErrorInvalidValue;
   }
+}
+
+cudaError_t launch_trace(const TraceArgs &a, uint32_t logN, cudaStream_t s) { return launch_mode<false>(a, logN, s); }
+
+cudaError_t launch_plaintext_mul(const TraceArgs &a, uint32_t logN, cudaStream_t s) {
+  return launch_mode<true>(a, logN, s);
 }
 
 }  // namespace rosetta

@@ -175,3 +175,62 @@ def test_trace_argument_checks():
     with pytest.raises(R.RosettaError) as e:
         big.upload_trace_keys(G.to_dev(np.zeros((13, 2, 2, 8192), np.uint64)), 16, 2)
     assert e.value.status == -2                     # N = 8192 not supported for the trace
+
+
+# ------------------------------------------------------------------ plaintext x ciphertext
+
+@pytest.mark.parametrize("name,batch,full_range,with_q", [
+    ("tiny", 7, True, True), ("standard", 5, True, False), ("standard", 3, False, True), ("gpt2_mlp", 3, True, True)])
+def test_plaintext_mul_bitexact(name, batch, full_range, with_q):
+    """(P * A, P * B + Q) word for word against the oracle; P over all of int64
+    or small, Q random or absent, a ragged batch."""
+    p = W.CONFIGS[name]
+    g = np.random.default_rng(batch + p.N)
+    if full_range:
+        P = g.integers(-2**63, 2**63, size=p.N, dtype=np.int64)
+    else:
+        P = g.integers(-1000, 1001, size=p.N, dtype=np.int64)
+    Qv = W.uniform_u64((p.N,), W.rng(p.seed, "sample", 61)) if with_q else None
+    glwe = W.uniform_u64((batch, 2, p.N), W.rng(p.seed, "sample", 60))
+    import paper_2609_16915_gb300 as R
+    ctx = R.Context(p)
+    out = G.empty_dev(batch, 2, p.N)
+    ctx.plaintext_mul_batch(G.to_dev(glwe), P, out, plain_add=Qv)
+    ctx.sync_status()
+    assert np.array_equal(G.to_host(out), O.plaintext_mul_batch(glwe, P, Qv))
+
+
+def test_plaintext_mul_device_q_and_reuse():
+    """Q from device memory; a second call with another P reuses the staged rows."""
+    p = W.CONFIGS["standard"]
+    g = np.random.default_rng(9)
+    glwe = W.uniform_u64((2, 2, p.N), W.rng(p.seed, "sample", 62))
+    Qv = W.uniform_u64((p.N,), W.rng(p.seed, "sample", 63))
+    import paper_2609_16915_gb300 as R
+    ctx = R.Context(p)
+    for _ in range(2):
+        P = g.integers(-2**20, 2**20, size=p.N, dtype=np.int64)
+        out = G.empty_dev(2, 2, p.N)
+        ctx.plaintext_mul_batch(G.to_dev(glwe), P, out, plain_add=G.to_dev(Qv))
+        ctx.sync_status()
+        assert np.array_equal(G.to_host(out), O.plaintext_mul_batch(glwe, P, Qv))
+
+
+def test_plaintext_mul_argument_checks():
+    import paper_2609_16915_gb300 as R
+    p = W.CONFIGS["standard"]
+    ctx = R.Context(p)
+    P = np.zeros(p.N, np.int64)
+    with pytest.raises(R.RosettaError) as e:        # host ciphertexts
+        ctx.plaintext_mul_batch(np.zeros((1, 2, p.N), np.uint64), P, G.empty_dev(1, 2, p.N))
+    assert e.value.status == -1
+    with pytest.raises(R.RosettaError) as e:        # device P
+        ctx.plaintext_mul_batch(G.to_dev(np.zeros((1, 2, p.N), np.uint64)), G.to_dev(P.view(np.uint64)),
+                                G.empty_dev(1, 2, p.N))
+    assert e.value.status == -1
+    big = R.Context(W.CONFIGS["llama_silu"])
+    N8 = W.CONFIGS["llama_silu"].N
+    with pytest.raises(R.RosettaError) as e:
+        big.plaintext_mul_batch(G.to_dev(np.zeros((1, 2, N8), np.uint64)), np.zeros(N8, np.int64),
+                                G.empty_dev(1, 2, N8))
+    assert e.value.status == -2

@@ -438,3 +438,51 @@ def test_trace_real_keys_isolates_constant_term():
     bound = per_step * (2 ** steps)
     assert max(abs(e) for e in err) < bound
     assert bound < (1 << 52) * N // 2     # the bound itself leaves the message readable
+
+
+# ------------------------------------------------------------------ plaintext x ciphertext
+
+@pytest.mark.parametrize("N", [1, 4, 16])
+def test_plaintext_mul_matches_integer_convolution(N):
+    """(P * A, P * B + Q) with P signed: each component an exact integer
+    negacyclic convolution reduced mod 2^64 (the linear mapping of the
+    lookup protocol, Cryptographic Lookup Protocol, Steps 2 and 3)."""
+    rs = random.Random(100 + N)
+    for with_q in (False, True):
+        P = [rs.randrange(-2**63, 2**63) for _ in range(N)]
+        c = [[rs.getrandbits(64) for _ in range(N)] for _ in range(2)]
+        q = [rs.getrandbits(64) for _ in range(N)]
+        want = []
+        for comp in range(2):
+            w = [0] * N
+            for i in range(N):
+                for j in range(N):
+                    t = i + j
+                    w[t % N] += (P[i] * c[comp][j]) * (-1 if t >= N else 1)
+            if comp == 1 and with_q:
+                w = [w[t] + q[t] for t in range(N)]
+            want.append([x % Q for x in w])
+        got = O.plaintext_mul_batch(np.array([c], np.uint64), np.array(P, np.int64),
+                                    np.array(q, np.uint64) if with_q else None)
+        assert [[int(x) for x in row] for row in got[0]] == want
+
+
+def test_plaintext_mul_scales_the_phase():
+    """phase(P * c) = P * phase(c): the product by a plaintext acts on the
+    encrypted message (noiseless encryption of m under S)."""
+    N = 64
+    g = np.random.default_rng(5)
+    S = g.integers(0, 2, size=(1, N), dtype=np.uint64)
+    A = g.integers(0, 2**64, size=(1, N), dtype=np.uint64, endpoint=False)
+    m = (g.integers(0, 16, size=N, dtype=np.uint64) << np.uint64(58))
+    glwe = O.glwe_encrypt(S, m, A, np.zeros(N, np.uint64))
+    P = g.integers(-3, 4, size=N)
+    got = O.plaintext_mul_batch(glwe.reshape(1, 2, N), P)[0]
+    ph = O.glwe_phase(S, got)
+    # P * m by hand: negacyclic, small P
+    want = [0] * N
+    for i in range(N):
+        for j in range(N):
+            t = i + j
+            want[t % N] += int(P[i]) * int(m[j]) * (-1 if t >= N else 1)
+    assert [int(x) for x in ph] == [x % Q for x in want]

@@ -194,6 +194,42 @@ int rosetta_trace_batch(rosetta_ctx *ctx, const uint64_t *glwe_in, uint32_t batc
 int rosetta_plaintext_mul_batch(rosetta_ctx *ctx, const uint64_t *glwe_in, uint32_t batch, const int64_t *plain_mul,
                                 const uint64_t *plain_add, uint64_t *glwe_out, void *stream);
 
+/* Tables of one segmented lookup (Segmented LUT Evaluation; Cryptographic
+ * Lookup Protocol, Steps 2 and 3), k = 1, N <= 4096, encoded by the caller as
+ * integer polynomials (all HOST memory, copied; the call returns when the
+ * tables are resident):
+ *   p_hat [N] int64, q_hat [N] uint64   -- index polynomials p(X), q(X)
+ *   a_hat [n_seg][N] int64, b_hat [n_seg][N] uint64 -- per-segment slope and
+ *                                          offset polynomials a_s(X), b_s(X)
+ * "Coefficient" s of a polynomial selected by an encrypted index is the box of
+ * coefficients a blind rotation by that index can land on: the caller lays
+ * out p, q with N / n_seg coefficients per segment and a_s, b_s with
+ * N / N_br per interval, each pre-rotated by half a box, the half box below 0
+ * negated (as the LUT test polynomial).  n_seg: power of two, 1 .. 256.
+ * Replaces any previous tables.  Errors: INVALID_ARG, UNSUPPORTED_PARAMS, CUDA,
+ * OOM. */
+int rosetta_upload_lookup_table(rosetta_ctx *ctx, uint32_t n_seg, const int64_t *p_hat, const uint64_t *q_hat,
+                                const int64_t *a_hat, const uint64_t *b_hat, void *stream);
+
+/* Encrypted segmented lookup f(x) ~ a_SI x + b_SI (Cryptographic Lookup
+ * Protocol, Steps 2 and 3; the segment index S comes from the comparisons of
+ * Step 1, which are not part of this library):
+ *   Step 2: [[t]] = p [[x]] + q; [[I]] = KS(extract(BlindRot([[t]], [[S]])));
+ *   Step 3: r_s = Trace(BlindRot(a_s [[x]] + b_s, [[I]])) for every segment s;
+ *           R = Box_0 sum_s X^(s N/n_seg) r_s; out = Trace(BlindRot(R, [[S]])).
+ *   glwe_x  [batch][2][N] uint64: x in the constant coefficient of the message
+ *           (the other message coefficients zero), device memory
+ *   lwe_seg [batch][n+1] uint64: LWE of S with Delta = 2^(63 - log2 n_seg), device
+ *   glwe_out [batch][2][N] uint64, device, no overlap with the inputs: the phase's
+ *           constant coefficient is N^2 (a_SI x + b_SI) in the caller's scale, the
+ *           others ~ 0 (each Trace multiplies by N: N has no inverse mod 2^64)
+ * Needs the BSK, KSK, trace keys and lookup tables.  Stream-ordered, no host
+ * synchronisation.  Per ciphertext: n_seg + 2 plaintext products, n_seg + 2
+ * blind rotations, one key switch, n_seg + 1 traces.  Errors: INVALID_ARG,
+ * KEYS_MISSING, CUDA, OOM. */
+int rosetta_segmented_lookup_batch(rosetta_ctx *ctx, const uint64_t *glwe_x, const uint64_t *lwe_seg, uint32_t batch,
+                                   uint64_t *glwe_out, void *stream);
+
 /* Same computation and result as rosetta_pbs_batch, for callers that cannot
  * allocate device memory during the call (their device memory belongs to
  * another allocator, or their serving loop forbids allocation after

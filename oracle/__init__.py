@@ -395,3 +395,51 @@ def keyswitch_batch(p, ksk, lwe_big, threads=None) -> np.ndarray:
     with ThreadPoolExecutor(threads or default_threads()) as ex:
         list(ex.map(one, range(lwe_big.shape[0])))
     return out
+
+
+# ---------------------------------------------------------------- encrypted segmented lookup (k = 1)
+
+def segment_box(s: int, n_seg: int, N: int) -> np.ndarray:
+    """[N] int64: +1 on the coefficients s N/n_seg + d, -h <= d < h (h half a
+    box), the ones below 0 wrapped to N + d with a minus sign (X^N = -1)."""
+    box = N // n_seg
+    h = box // 2
+    v = np.zeros(N, np.int64)
+    for d in range(-h, box - h):
+        j = s * box + d
+        if j < 0:
+            v[j + N] = -1
+        else:
+            v[j] = 1
+    return v
+
+
+def segmented_lookup_batch(p, bsk, ksk, tkeys, t_base_log: int, t_level: int, glwe_x, lwe_seg,
+                           p_hat, q_hat, a_hat, b_hat, threads=None) -> np.ndarray:
+    """[batch][2][N]: the encrypted lookup of the Cryptographic Lookup
+    Protocol, Steps 2 and 3, for each [[x]] (glwe_x) and segment index [[S]]
+    (lwe_seg), with the caller's integer tables.
+      Step 2: [[t]] = p [[x]] + q; PBS([[t]], [[S]]) (blind rotation,
+              extraction of the constant term, key switch) = [[I]].
+      Step 3, phase 1: [[r_s]] = a_s [[x]] + b_s; r_s = Trace(BlindRot(r_s, [[I]])).
+      Phase 2: [[R]] = sum_s r_s X^s, the s-th coefficient being the segment
+              box of s (so r_s times the box polynomial);
+              out = Trace(BlindRot([[R]], [[S]]))."""
+    glwe_x = _c(glwe_x)
+    lwe_seg = _c(np.atleast_2d(lwe_seg))
+    batch, _, N = glwe_x.shape
+    n_seg = a_hat.shape[0]
+    # Step 2
+    t = plaintext_mul_batch(glwe_x, p_hat, q_hat)
+    t_rot = blind_rotate_glwe_batch(p, bsk, lwe_seg, t, threads)
+    lwe_I = keyswitch_batch(p, ksk, np.stack([sample_extract(g) for g in t_rot]), threads)
+    # Step 3, phase 1 (all segments of all ciphertexts at once)
+    r = np.concatenate([plaintext_mul_batch(glwe_x, a_hat[s], b_hat[s]) for s in range(n_seg)])
+    r = blind_rotate_glwe_batch(p, bsk, np.tile(lwe_I, (n_seg, 1)), r, threads)
+    r = trace_batch(tkeys, r, t_base_log, t_level, threads).reshape(n_seg, batch, 2, N)
+    # phase 2
+    R = np.zeros((batch, 2, N), np.uint64)
+    for s in range(n_seg):
+        R += plaintext_mul_batch(r[s], segment_box(s, n_seg, N))
+    R_rot = blind_rotate_glwe_batch(p, bsk, lwe_seg, R, threads)
+    return trace_batch(tkeys, R_rot, t_base_log, t_level, threads)

@@ -23,7 +23,7 @@ STATUS = {0: "ok", -1: "invalid argument", -2: "unsupported parameters", -3: "ke
 EXPORTS = ("rosetta_params_init", "rosetta_upload_bsk", "rosetta_upload_ksk", "rosetta_pbs_batch",
            "rosetta_blind_rotate_extract_batch", "rosetta_keyswitch_batch", "rosetta_pbs_batch_multi_lut",
            "rosetta_blind_rotate_glwe_batch", "rosetta_upload_trace_keys", "rosetta_trace_batch",
-           "rosetta_plaintext_mul_batch",
+           "rosetta_plaintext_mul_batch", "rosetta_upload_lookup_table", "rosetta_segmented_lookup_batch",
            "rosetta_pbs_batch_noalloc",
            "rosetta_sync_status", "rosetta_destroy", "rosetta_status_string")
 
@@ -64,6 +64,8 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     L.rosetta_upload_trace_keys.argtypes = [vp, u64p, ctypes.c_size_t, u32, u32, ctypes.c_int, vp]
     L.rosetta_trace_batch.argtypes = [vp, u64p, u32, u64p, vp]
     L.rosetta_plaintext_mul_batch.argtypes = [vp, u64p, u32, u64p, u64p, u64p, vp]
+    L.rosetta_upload_lookup_table.argtypes = [vp, u32, u64p, u64p, u64p, u64p, vp]
+    L.rosetta_segmented_lookup_batch.argtypes = [vp, u64p, u64p, u32, u64p, vp]
     L.rosetta_sync_status.argtypes = [vp, vp]
     L.rosetta_destroy.argtypes = [vp]
     L.rosetta_destroy.restype = None
@@ -206,6 +208,25 @@ class Context:
                                                   _stream(stream)))
         return glwe_out
 
+    def rosetta_upload_lookup_table(self, p_hat, q_hat, a_hat, b_hat, stream=None):
+        """Host tables of one segmented lookup: p_hat, q_hat [N]; a_hat, b_hat [n_seg][N]."""
+        n = self.params.N
+        n_seg = a_hat.shape[0]
+        for name, v, shape in (("p_hat", p_hat, (n,)), ("q_hat", q_hat, (n,)), ("a_hat", a_hat, (n_seg, n)),
+                               ("b_hat", b_hat, (n_seg, n))):
+            if v.shape != shape or v.dtype.itemsize != 8:
+                raise ValueError(f"{name} must be 64-bit words of shape {shape}")
+        _check("rosetta_upload_lookup_table",
+               load().rosetta_upload_lookup_table(self._h, n_seg, _ptr(p_hat), _ptr(q_hat), _ptr(a_hat), _ptr(b_hat),
+                                                  _stream(stream)))
+
+    def rosetta_segmented_lookup_batch(self, glwe_x, lwe_seg, glwe_out, stream=None):
+        """Encrypted segmented lookup of each [[x]] (glwe_x [batch][2][N]) with segment index lwe_seg [batch][n+1]."""
+        _check("rosetta_segmented_lookup_batch",
+               load().rosetta_segmented_lookup_batch(self._h, _ptr(glwe_x), _ptr(lwe_seg), glwe_x.shape[0],
+                                                     _ptr(glwe_out), _stream(stream)))
+        return glwe_out
+
     def rosetta_pbs_batch_noalloc(self, lwe_in, lut, lwe_out, stream=None):
         """rosetta_pbs_batch without any device allocation in the call (fixed
         in-library scratch; device buffers only, bounded batch)."""
@@ -228,4 +249,6 @@ class Context:
     upload_trace_keys = rosetta_upload_trace_keys
     trace_batch = rosetta_trace_batch
     plaintext_mul_batch = rosetta_plaintext_mul_batch
+    upload_lookup_table = rosetta_upload_lookup_table
+    segmented_lookup_batch = rosetta_segmented_lookup_batch
     sync_status = rosetta_sync_status

@@ -34,4 +34,14 @@ struct rosetta_ctx {
   uint64_t *d_pm_raw = nullptr;   // plaintext-multiply gadget rows, raw [8][2][N]
   uint32_t *d_pm_key = nullptr;   // the same in the transform domain
   uint64_t *d_pm_add = nullptr;   // staged additive plaintext [N]
+  // segmented lookup: plaintext polynomials (P, A_0..A_{n_seg-1}, Box_0) as gadget rows in the
+  // transform domain [n_seg+2][prime][8][2][N], additive ones (Q, B_0..B_{n_seg-1}) [n_seg+1][N]
+  uint32_t *d_lk_key = nullptr;
+  uint64_t *d_lk_add = nullptr;
+  uint32_t lk_nseg = 0;
+  bool have_lk = false;
+  uint64_t *d_lk_t = nullptr, *d_lk_u = nullptr, *d_lk_R = nullptr;  // [batch][2][N] each
+  size_t lk_t_cap = 0, lk_u_cap = 0, lk_R_cap = 0;
+  uint64_t *d_lk_I = nullptr;     // interval-index LWEs [batch][n+1]
+  size_t lk_I_cap = 0;
 };

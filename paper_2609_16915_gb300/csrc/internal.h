@@ -78,6 +78,8 @@ cudaError_t launch_key_transform(const uint64_t *raw, uint32_t *out, const uint2
 size_t trace_smem_bytes(uint32_t logN, uint32_t level);
 cudaError_t launch_trace(const TraceArgs &a, uint32_t logN, cudaStream_t s);
 cudaError_t launch_plaintext_mul(const TraceArgs &a, uint32_t logN, cudaStream_t s);
+cudaError_t launch_monomial_acc(uint64_t *R, const uint64_t *r, uint32_t count, uint32_t logN, uint32_t e, bool first,
+                                cudaStream_t s);
 cudaError_t launch_ksk_corr(const uint64_t *ksk, uint64_t *corr, uint32_t rows, uint32_t n, uint32_t base_log,
                             cudaStream_t s);
 

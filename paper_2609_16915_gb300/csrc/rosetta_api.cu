@@ -184,6 +184,48 @@ KsArgs ks_args(const rosetta_ctx *c, const uint64_t *big, uint32_t batch, uint64
   return k;
 }
 
+// Plaintext products use an exact 64-bit gadget (16 bits x 4 levels) against
+// noiseless rows: row comp*4 + l of component comp holds P 2^(64 - (l+1) 16),
+// the other component 0 (raw layout [8][2][N]).
+constexpr uint32_t kPmBase = 16, kPmLev = 4, kPmRows = 2 * kPmLev;
+
+void pm_rows(uint64_t *raw, const int64_t *P, size_t N) {
+  for (size_t w = 0; w < kPmRows * 2 * N; ++w) raw[w] = 0;
+  for (uint32_t comp = 0; comp < 2; ++comp)
+    for (uint32_t l = 0; l < kPmLev; ++l)
+      for (size_t t = 0; t < N; ++t)
+        raw[((comp * kPmLev + l) * 2 + comp) * N + t] = static_cast<uint64_t>(P[t]) << (64 - (l + 1) * kPmBase);
+}
+
+// out[b] = (P * in_A, P * in_B + add) with P given by its transformed gadget rows.
+cudaError_t launch_pm(const rosetta_ctx *c, const uint32_t *key, const uint64_t *add, const uint64_t *in,
+                      uint32_t batch, uint64_t *out, cudaStream_t s) {
+  TraceArgs a{};
+  a.glwe_in = in;
+  a.glwe_out = out;
+  a.keys = key;
+  a.plain_add = add;
+  a.tw = c->d_tw;
+  a.base_log = kPmBase;
+  a.level = kPmRows;
+  a.batch = batch;
+  a.cc = c->cc;
+  return launch_plaintext_mul(a, c->logN, s);
+}
+
+TraceArgs trace_args(const rosetta_ctx *c, const uint64_t *in, uint32_t batch, uint64_t *out) {
+  TraceArgs a{};
+  a.glwe_in = in;
+  a.glwe_out = out;
+  a.keys = c->d_trk;
+  a.tw = c->d_tw;
+  a.base_log = c->trk_base_log;
+  a.level = c->trk_level;
+  a.batch = batch;
+  a.cc = c->cc;
+  return a;
+}
+
 }  // namespace
 
 extern "C" {
@@ -478,16 +520,7 @@ int rosetta_trace_batch(rosetta_ctx *c, const uint64_t *glwe_in, uint32_t batch,
   if (!is_device_ptr(glwe_in) || !is_device_ptr(glwe_out) || !aligned8(glwe_in) || !aligned8(glwe_out) ||
       overlaps(glwe_in, gbytes, glwe_out, gbytes))
     return ROSETTA_ERR_INVALID_ARG;
-  TraceArgs a{};
-  a.glwe_in = glwe_in;
-  a.glwe_out = glwe_out;
-  a.keys = c->d_trk;
-  a.tw = c->d_tw;
-  a.base_log = c->trk_base_log;
-  a.level = c->trk_level;
-  a.batch = batch;
-  a.cc = c->cc;
-  cudaError_t e = launch_trace(a, c->logN, as_stream(stream));
+  cudaError_t e = launch_trace(trace_args(c, glwe_in, batch, glwe_out), c->logN, as_stream(stream));
   return e == cudaSuccess ? ROSETTA_OK : cuda_fail(e);
 }
 
@@ -504,13 +537,8 @@ int rosetta_plaintext_mul_batch(rosetta_ctx *c, const uint64_t *glwe_in, uint32_
       !aligned8(plain_mul) || (plain_add && !aligned8(plain_add)) || overlaps(glwe_in, gbytes, glwe_out, gbytes))
     return ROSETTA_ERR_INVALID_ARG;
   if (is_device_ptr(plain_mul)) return ROSETTA_ERR_INVALID_ARG;  // the gadget rows are built on the host
-  // noiseless gadget rows: row c*4 + l of component c is P 2^(64 - (l+1) 16)
-  constexpr uint32_t kBase = 16, kLev = 4, kRows = 2 * kLev;
-  std::vector<uint64_t> raw(kRows * 2 * N, 0);
-  for (uint32_t comp = 0; comp < 2; ++comp)
-    for (uint32_t l = 0; l < kLev; ++l)
-      for (size_t t = 0; t < N; ++t)
-        raw[((comp * kLev + l) * 2 + comp) * N + t] = static_cast<uint64_t>(plain_mul[t]) << (64 - (l + 1) * kBase);
+  std::vector<uint64_t> raw(kPmRows * 2 * N);
+  pm_rows(raw.data(), plain_mul, N);
   cudaStream_t s = as_stream(stream);
   cudaError_t e = cudaSuccess;
   if (!c->d_pm_raw) e = cudaMalloc(&c->d_pm_raw, raw.size() * 8);
@@ -520,21 +548,118 @@ int rosetta_plaintext_mul_batch(rosetta_ctx *c, const uint64_t *glwe_in, uint32_
   e = cudaMemcpyAsync(c->d_pm_raw, raw.data(), raw.size() * 8, cudaMemcpyHostToDevice, s);
   if (e == cudaSuccess && plain_add)
     e = cudaMemcpyAsync(c->d_pm_add, plain_add, N * 8, cudaMemcpyDefault, s);
-  if (e == cudaSuccess) e = launch_key_transform(c->d_pm_raw, c->d_pm_key, c->d_tw, c->cc, c->logN, 1, kRows, s);
-  if (e != cudaSuccess) return cuda_fail(e);
-  TraceArgs a{};
-  a.glwe_in = glwe_in;
-  a.glwe_out = glwe_out;
-  a.keys = c->d_pm_key;
-  a.plain_add = plain_add ? c->d_pm_add : nullptr;
-  a.tw = c->d_tw;
-  a.base_log = kBase;
-  a.level = kRows;
-  a.batch = batch;
-  a.cc = c->cc;
-  e = launch_plaintext_mul(a, c->logN, s);
+  if (e == cudaSuccess) e = launch_key_transform(c->d_pm_raw, c->d_pm_key, c->d_tw, c->cc, c->logN, 1, kPmRows, s);
+  if (e == cudaSuccess) e = launch_pm(c, c->d_pm_key, plain_add ? c->d_pm_add : nullptr, glwe_in, batch, glwe_out, s);
   if (e != cudaSuccess) return cuda_fail(e);
   e = cudaStreamSynchronize(s);  // the host staging vector goes out of scope
+  return e == cudaSuccess ? ROSETTA_OK : cuda_fail(e);
+}
+
+int rosetta_upload_lookup_table(rosetta_ctx *c, uint32_t n_seg, const int64_t *p_hat, const uint64_t *q_hat,
+                                const int64_t *a_hat, const uint64_t *b_hat, void *stream) {
+  if (!c || !p_hat || !q_hat || !a_hat || !b_hat) return ROSETTA_ERR_INVALID_ARG;
+  const size_t N = c->prm.poly_size;
+  if (c->logN > 12 || c->prm.glwe_dim != 1) return ROSETTA_ERR_UNSUPPORTED_PARAMS;
+  if (n_seg == 0 || n_seg > 256 || (n_seg & (n_seg - 1)) || n_seg > N) return ROSETTA_ERR_UNSUPPORTED_PARAMS;
+  if (is_device_ptr(p_hat) || is_device_ptr(q_hat) || is_device_ptr(a_hat) || is_device_ptr(b_hat))
+    return ROSETTA_ERR_INVALID_ARG;  // the tables are encoded on the host
+  if (cudaSetDevice(c->device) != cudaSuccess) return ROSETTA_ERR_CUDA;
+  const uint32_t polys = n_seg + 2;  // P, A_0 .. A_{n_seg-1}, Box_0
+  const size_t poly_words = kPmRows * 2 * N;
+  std::vector<uint64_t> raw(polys * poly_words);
+  pm_rows(raw.data(), p_hat, N);
+  for (uint32_t sg = 0; sg < n_seg; ++sg) pm_rows(raw.data() + (1 + sg) * poly_words, a_hat + sg * N, N);
+  // Box_0: the coefficients a rotation by less than half a segment box brings to
+  // position 0 (+1 on [0, h), -1 on [N - h, N) by X^N = -1), h = N / (2 n_seg)
+  std::vector<int64_t> box(N, 0);
+  const size_t h = N / n_seg / 2;
+  box[0] = 1;
+  for (size_t t = 1; t < h; ++t) box[t] = 1;
+  for (size_t t = N - h; t < N; ++t) box[t] = -1;
+  pm_rows(raw.data() + (1 + n_seg) * poly_words, box.data(), N);
+  std::vector<uint64_t> add((1 + n_seg) * N);
+  for (size_t t = 0; t < N; ++t) add[t] = q_hat[t];
+  for (size_t w = 0; w < n_seg * N; ++w) add[N + w] = b_hat[w];
+
+  cudaStream_t s = as_stream(stream);
+  cudaError_t e = cudaStreamSynchronize(s);  // no lookup in flight reads the old tables
+  uint64_t *d_raw = nullptr;
+  if (e == cudaSuccess) e = cudaMalloc(&d_raw, raw.size() * 8);
+  if (e != cudaSuccess) return cuda_fail(e);
+  cudaFree(c->d_lk_key);
+  cudaFree(c->d_lk_add);
+  c->d_lk_key = nullptr;
+  c->d_lk_add = nullptr;
+  c->have_lk = false;
+  e = cudaMalloc(&c->d_lk_key, raw.size() * kPrimes * sizeof(uint32_t));
+  if (e == cudaSuccess) e = cudaMalloc(&c->d_lk_add, add.size() * 8);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(d_raw, raw.data(), raw.size() * 8, cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(c->d_lk_add, add.data(), add.size() * 8, cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess) e = launch_key_transform(d_raw, c->d_lk_key, c->d_tw, c->cc, c->logN, polys, kPmRows, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  cudaFree(d_raw);
+  if (e != cudaSuccess) return cuda_fail(e);
+  c->lk_nseg = n_seg;
+  c->have_lk = true;
+  return ROSETTA_OK;
+}
+
+int rosetta_segmented_lookup_batch(rosetta_ctx *c, const uint64_t *glwe_x, const uint64_t *lwe_seg, uint32_t batch,
+                                   uint64_t *glwe_out, void *stream) {
+  if (!c) return ROSETTA_ERR_INVALID_ARG;
+  if (batch == 0) return ROSETTA_OK;
+  if (!glwe_x || !lwe_seg || !glwe_out) return ROSETTA_ERR_INVALID_ARG;
+  if (!c->have_bsk || !c->have_ksk || !c->have_trk || !c->have_lk) return ROSETTA_ERR_KEYS_MISSING;
+  if (cudaSetDevice(c->device) != cudaSuccess) return ROSETTA_ERR_CUDA;
+  const size_t N = c->prm.poly_size, gw = 2 * N;
+  const size_t gbytes = (size_t)batch * gw * 8, lbytes = (size_t)batch * lwe_words(c) * 8;
+  if (!is_device_ptr(glwe_x) || !is_device_ptr(lwe_seg) || !is_device_ptr(glwe_out) || !aligned8(glwe_x) ||
+      !aligned8(lwe_seg) || !aligned8(glwe_out) || overlaps(glwe_x, gbytes, glwe_out, gbytes) ||
+      overlaps(lwe_seg, lbytes, glwe_out, gbytes))
+    return ROSETTA_ERR_INVALID_ARG;
+  cudaStream_t s = as_stream(stream);
+  int r = ensure(&c->d_lk_t, &c->lk_t_cap, batch * gw, s);
+  if (r == ROSETTA_OK) r = ensure(&c->d_lk_u, &c->lk_u_cap, batch * gw, s);
+  if (r == ROSETTA_OK) r = ensure(&c->d_lk_R, &c->lk_R_cap, batch * gw, s);
+  if (r == ROSETTA_OK) r = ensure(&c->d_lk_I, &c->lk_I_cap, batch * lwe_words(c), s);
+  if (r == ROSETTA_OK) r = ensure_big(c, batch, s);
+  if (r != ROSETTA_OK) return r;
+  const uint32_t nseg = c->lk_nseg;
+  const size_t key_words = (size_t)kPrimes * kPmRows * gw;
+  const uint32_t *kP = c->d_lk_key, *kBox = c->d_lk_key + (1 + nseg) * key_words;
+  uint64_t *T = c->d_lk_t, *U = c->d_lk_u, *R = c->d_lk_R, *I = c->d_lk_I;
+
+  // Step 2: t = p(X) [[x]] + q(X); PBS of t selected by [[S]] gives [[I]]
+  cudaError_t e = launch_pm(c, kP, c->d_lk_add, glwe_x, batch, T, s);
+  if (e == cudaSuccess) {
+    BrArgs a = br_args(c, lwe_seg, batch, nullptr, c->d_big);
+    a.glwe_in = T;
+    e = launch_blind_rotate(a, c->logN, c->dig16, s);
+  }
+  if (e == cudaSuccess) e = launch_keyswitch(ks_args(c, c->d_big, batch, I), s);
+  // Step 3, phase 1: r_s = a_s(X) [[x]] + b_s(X), rotated by [[I]], traced, and
+  // accumulated as R = sum_s X^(s box) r_s
+  const uint32_t seg_box = static_cast<uint32_t>(N / nseg);
+  for (uint32_t sg = 0; sg < nseg && e == cudaSuccess; ++sg) {
+    e = launch_pm(c, c->d_lk_key + (1 + sg) * key_words, c->d_lk_add + (1 + sg) * N, glwe_x, batch, T, s);
+    if (e == cudaSuccess) {
+      BrArgs a = br_args(c, I, batch, nullptr, nullptr);
+      a.glwe_in = T;
+      a.glwe_out = U;
+      e = launch_blind_rotate(a, c->logN, c->dig16, s);
+    }
+    if (e == cudaSuccess) e = launch_trace(trace_args(c, U, batch, T), c->logN, s);
+    if (e == cudaSuccess) e = launch_monomial_acc(R, T, 2 * batch, c->logN, sg * seg_box, sg == 0, s);
+  }
+  // phase 2: spread each value over its segment box, rotate by [[S]], trace
+  if (e == cudaSuccess) e = launch_pm(c, kBox, nullptr, R, batch, T, s);
+  if (e == cudaSuccess) {
+    BrArgs a = br_args(c, lwe_seg, batch, nullptr, nullptr);
+    a.glwe_in = T;
+    a.glwe_out = U;
+    e = launch_blind_rotate(a, c->logN, c->dig16, s);
+  }
+  if (e == cudaSuccess) e = launch_trace(trace_args(c, U, batch, glwe_out), c->logN, s);
   return e == cudaSuccess ? ROSETTA_OK : cuda_fail(e);
 }
 
@@ -569,6 +694,12 @@ void rosetta_destroy(rosetta_ctx *c) {
   cudaFree(c->d_pm_raw);
   cudaFree(c->d_pm_key);
   cudaFree(c->d_pm_add);
+  cudaFree(c->d_lk_key);
+  cudaFree(c->d_lk_add);
+  cudaFree(c->d_lk_t);
+  cudaFree(c->d_lk_u);
+  cudaFree(c->d_lk_R);
+  cudaFree(c->d_lk_I);
   delete c;
 }
 

@@ -262,4 +262,32 @@ cudaError_t launch_plaintext_mul(const TraceArgs &a, uint32_t logN, cudaStream_t
   return launch_mode<true>(a, logN, s);
 }
 
+// R <- (first ? 0 : R) + X^e r for `count` polynomials of N words (0 <= e < N):
+// coefficient j of X^e r is r[j - e] for j >= e and -r[j - e + N] below.
+__global__ void __launch_bounds__(256) monomial_acc_kernel(uint64_t *__restrict__ R, const uint64_t *__restrict__ r,
+                                                          size_t words, uint32_t logN, uint32_t e, bool first) {
+  const uint32_t N = 1u << logN;
+  const size_t stride = static_cast<size_t>(gridDim.x) * blockDim.x;
+  for (size_t i = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < words; i += stride) {
+    const uint32_t j = static_cast<uint32_t>(i) & (N - 1);
+    const size_t row = i - j;
+    const uint64_t v = j >= e ? r[row + j - e] : 0ull - r[row + j - e + N];
+    R[i] = first ? v : R[i] + v;
+  }
+}
+
+cudaError_t launch_monomial_acc(uint64_t *R, const uint64_t *r, uint32_t count, uint32_t logN, uint32_t e, bool first,
+                                cudaStream_t s) {
+  const size_t words = static_cast<size_t>(count) << logN;
+  if (words == 0) return cudaSuccess;
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  size_t blocks = (words + 255) / 256;
+  const size_t cap = static_cast<size_t>(sms > 0 ? sms : 1) * 8;
+  if (blocks > cap) blocks = cap;
+  monomial_acc_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(R, r, words, logN, e, first);
+  return cudaGetLastError();
+}
+
 }  // namespace rosetta

@@ -15,6 +15,16 @@ the candidate values.
 Each interval's line interpolates f at the interval's two Chebyshev nodes
 c +- (h/2) cos(pi/4) (c its centre, h its width): the near-minimax linear
 fit, and the one that reproduces the paper's printed coefficients.
+
+``encode`` turns a table into the integer polynomials the encrypted lookup
+(``rosetta_segmented_lookup_batch``) takes.  A "coefficient" selected by an
+encrypted index is a box of N/K ring coefficients (K = N_seg or N_br), laid
+out like a LUT test polynomial: pre-rotated by half a box, the half box below
+position 0 negated (X^N = -1), so that a blind rotation by the index, noise
+included, lands inside the right box.  The interval index I is carried at
+Delta_I = 2^(63 - log2 N_br) per interval with half an interval subtracted,
+so that the rounding of the next blind rotation's modulus switch takes the
+floor of Step 2.
 """
 
 from __future__ import annotations
@@ -102,3 +112,79 @@ def index_polynomials(lut: SegmentedLUT):
 def value_polynomials(lut: SegmentedLUT, s: int):
     """Coefficients of a_s(X) = sum_i a_si X^i and b_s(X) = sum_i b_si X^i."""
     return lut.a[s].copy(), lut.b[s].copy()
+
+
+# ---------------------------------------------------------------- encrypted lookup tables
+
+def box_layout(values, N: int) -> list:
+    """[N] Python ints: values[i] on box i (N / len(values) coefficients),
+    pre-rotated by half a box, the half box below 0 holding -values[0]."""
+    K = len(values)
+    box = N // K
+    h = box // 2
+    return [values[(t + h) // box] if t < N - h else -values[0] for t in range(N)]
+
+
+@dataclass
+class EncodedLookup:
+    p_hat: np.ndarray      # [N] int64
+    q_hat: np.ndarray      # [N] uint64
+    a_hat: np.ndarray      # [N_seg][N] int64
+    b_hat: np.ndarray      # [N_seg][N] uint64
+    N: int
+    delta_x_log2: int      # x is carried as round(x 2^delta_x_log2)
+    delta_r_log2: int      # values a x + b before the traces, per unit
+
+
+def _pow2(v: int) -> bool:
+    return v > 0 and v & (v - 1) == 0
+
+
+def _i64(vals) -> np.ndarray:
+    if any(abs(v) >= 1 << 63 for v in vals):
+        raise ValueError("coefficient does not fit int64: lower the scales")
+    return np.array(vals, dtype=np.int64)
+
+
+def _u64(vals) -> np.ndarray:
+    return np.array([v % (1 << 64) for v in vals], dtype=np.uint64)
+
+
+def encode(lut: SegmentedLUT, N: int, delta_x_log2: int, delta_r_log2: int) -> EncodedLookup:
+    """Integer polynomials of Steps 2 and 3 for ring size N:
+    p, q with p_s = N_br/(tau_{s+1} - tau_s) Delta_I / Delta_x and
+    q_s = -tau_s N_br/(tau_{s+1} - tau_s) Delta_I - Delta_I / 2;
+    a_s, b_s with a_si Delta_r / Delta_x and b_si Delta_r per interval."""
+    if not (_pow2(lut.n_seg) and _pow2(lut.n_br) and lut.n_seg <= N and lut.n_br <= N):
+        raise ValueError("N_seg and N_br must be powers of two no larger than N")
+    d_i = 1 << (63 - (lut.n_br.bit_length() - 1))
+    w, q = index_polynomials(lut)
+    sx = 2.0 ** -delta_x_log2
+    p_vals = [round(float(w[s]) * d_i * sx) for s in range(lut.n_seg)]
+    q_vals = [round(float(q[s]) * d_i) - d_i // 2 for s in range(lut.n_seg)]
+    a_rows, b_rows = [], []
+    for s in range(lut.n_seg):
+        a_s, b_s = value_polynomials(lut, s)
+        a_rows.append(_i64(box_layout([round(float(v) * 2.0 ** (delta_r_log2 - delta_x_log2)) for v in a_s], N)))
+        b_rows.append(_u64(box_layout([round(float(v) * 2.0 ** delta_r_log2) for v in b_s], N)))
+    return EncodedLookup(_i64(box_layout(p_vals, N)), _u64(box_layout(q_vals, N)), np.stack(a_rows),
+                         np.stack(b_rows), N, delta_x_log2, delta_r_log2)
+
+
+def encode_x(x: float, delta_x_log2: int) -> int:
+    """Torus word carrying x in the constant coefficient of [[x]]."""
+    return round(x * 2.0 ** delta_x_log2) % (1 << 64)
+
+
+def segment_word(s: int, n_seg: int) -> int:
+    """Torus word carrying the segment index S of [[S]] (Delta = 2^(63 - log2 N_seg))."""
+    return (s << (63 - (n_seg.bit_length() - 1))) % (1 << 64)
+
+
+def decode(phase0: int, enc: EncodedLookup) -> float:
+    """f(x) from the constant coefficient of the lookup output's phase
+    (N^2 a_SI x + b_SI in units of 2^-delta_r_log2: each trace multiplies by N)."""
+    v = int(phase0) % (1 << 64)
+    if v >= 1 << 63:
+        v -= 1 << 64
+    return v / (enc.N * enc.N * 2.0 ** enc.delta_r_log2)

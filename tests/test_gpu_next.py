@@ -234,3 +234,98 @@ def test_plaintext_mul_argument_checks():
         big.plaintext_mul_batch(G.to_dev(np.zeros((1, 2, N8), np.uint64)), np.zeros(N8, np.int64),
                                 G.empty_dev(1, 2, N8))
     assert e.value.status == -2
+
+
+# ------------------------------------------------------------------ encrypted segmented lookup
+
+def _lookup_ctx(p, bsk, ksk, tk, tb, tl, tables):
+    ctx = G.make_ctx(p, bsk, ksk)
+    ctx.upload_trace_keys(G.to_dev(tk), tb, tl)
+    ctx.upload_lookup_table(*tables)
+    return ctx
+
+
+def test_lookup_bitexact_and_decrypts_small_ring():
+    """Real keys, the paper's 1/x table: GPU words = oracle words, and the
+    decryption is the cleartext segmented lookup (4.571 at x = 0.22)."""
+    from paper_2609_16915_gb300 import segmented as SG
+    from tests import lookup_util as LU
+    p = W.CONFIGS["lookup_small"]
+    keys = O.Keys(p, W.key_draws(p))
+    tk = LU.trace_keys(p, keys.glwe_key)
+    lut = LU.paper_table()
+    enc = SG.encode(lut, p.N, LU.DX, LU.DR)
+    xs = [0.22] + LU.sample_points(lut, 8, 11)
+    segs = [SG.segment_index(lut, x) for x in xs]
+    glwe, lwe = LU.encrypt_inputs(p, keys, xs, segs, lut.n_seg, sub=1)
+    tables = (enc.p_hat, enc.q_hat, enc.a_hat, enc.b_hat)
+    ctx = _lookup_ctx(p, keys.bsk, keys.ksk, tk, LU.TRACE_BASE_LOG, LU.TRACE_LEVEL, tables)
+    out = G.empty_dev(len(xs), 2, p.N)
+    ctx.segmented_lookup_batch(G.to_dev(glwe), G.to_dev(lwe), out)
+    ctx.sync_status()
+    got = G.to_host(out)
+    want = O.segmented_lookup_batch(p, keys.bsk, keys.ksk, tk, LU.TRACE_BASE_LOG, LU.TRACE_LEVEL, glwe, lwe, *tables)
+    assert np.array_equal(got, want)
+    S = keys.glwe_key.reshape(1, -1)
+    vals = [SG.decode(O.glwe_phase(S, got[b])[0], enc) for b in range(len(xs))]
+    assert vals[0] == pytest.approx(4.571, abs=2e-3)
+    for x, v in zip(xs, vals):
+        assert v == pytest.approx(SG.lookup(lut, x), abs=1e-2), x
+
+
+@pytest.mark.parametrize("n_seg", [1, 8])
+def test_lookup_bitexact_random_tables(n_seg):
+    """Random integer tables and uniform-word keys and inputs, other segment counts."""
+    p = W.CONFIGS["lookup_small"]
+    g = np.random.default_rng(40 + n_seg)
+    bsk, ksk = W.uniform_keys(p, seed=41)
+    tk = W.uniform_u64((p.N.bit_length() - 1, 4, 2, p.N), W.rng(p.seed, "sample", 80))
+    tables = (g.integers(-2**40, 2**40, size=p.N, dtype=np.int64), W.uniform_u64((p.N,), W.rng(p.seed, "sample", 81)),
+              g.integers(-2**40, 2**40, size=(n_seg, p.N), dtype=np.int64),
+              W.uniform_u64((n_seg, p.N), W.rng(p.seed, "sample", 82)))
+    glwe = W.uniform_u64((3, 2, p.N), W.rng(p.seed, "sample", 83))
+    lwe = W.uniform_u64((3, p.n + 1), W.rng(p.seed, "sample", 84))
+    ctx = _lookup_ctx(p, bsk, ksk, tk, 16, 4, tables)
+    out = G.empty_dev(3, 2, p.N)
+    ctx.segmented_lookup_batch(G.to_dev(glwe), G.to_dev(lwe), out)
+    ctx.sync_status()
+    assert np.array_equal(G.to_host(out), O.segmented_lookup_batch(p, bsk, ksk, tk, 16, 4, glwe, lwe, *tables))
+
+
+def test_lookup_bitexact_standard_ring():
+    """N = 2048, n = 742 (the bench's ring): one ciphertext, four segments,
+    sparse segment-index ciphertext (the oracle's cost)."""
+    p = W.CONFIGS["standard"]
+    g = np.random.default_rng(50)
+    bsk, ksk = W.uniform_keys(p, seed=51)
+    tk = W.uniform_u64((p.N.bit_length() - 1, 4, 2, p.N), W.rng(p.seed, "sample", 90))
+    n_seg = 4
+    tables = (g.integers(-2**40, 2**40, size=p.N, dtype=np.int64), W.uniform_u64((p.N,), W.rng(p.seed, "sample", 91)),
+              g.integers(-2**40, 2**40, size=(n_seg, p.N), dtype=np.int64),
+              W.uniform_u64((n_seg, p.N), W.rng(p.seed, "sample", 92)))
+    glwe = W.uniform_u64((1, 2, p.N), W.rng(p.seed, "sample", 93))
+    lwe = G.sparse_lwe(p, 1, 3, seed=9)
+    ctx = _lookup_ctx(p, bsk, ksk, tk, 16, 4, tables)
+    out = G.empty_dev(1, 2, p.N)
+    ctx.segmented_lookup_batch(G.to_dev(glwe), G.to_dev(lwe), out)
+    ctx.sync_status()
+    assert np.array_equal(G.to_host(out), O.segmented_lookup_batch(p, bsk, ksk, tk, 16, 4, glwe, lwe, *tables))
+
+
+def test_lookup_argument_checks():
+    import paper_2609_16915_gb300 as R
+    p = W.CONFIGS["lookup_small"]
+    bsk, ksk = W.uniform_keys(p, seed=42)
+    ctx = G.make_ctx(p, bsk, ksk)
+    glwe = G.to_dev(np.zeros((1, 2, p.N), np.uint64))
+    lwe = G.to_dev(np.zeros((1, p.n + 1), np.uint64))
+    with pytest.raises(R.RosettaError) as e:        # no trace keys, no tables
+        ctx.segmented_lookup_batch(glwe, lwe, G.empty_dev(1, 2, p.N))
+    assert e.value.status == -3
+    z64, zu = np.zeros(p.N, np.int64), np.zeros(p.N, np.uint64)
+    with pytest.raises(R.RosettaError) as e:        # 3 segments: not a power of two
+        ctx.upload_lookup_table(z64, zu, np.zeros((3, p.N), np.int64), np.zeros((3, p.N), np.uint64))
+    assert e.value.status == -2
+    with pytest.raises(R.RosettaError) as e:        # tables in device memory
+        ctx.upload_lookup_table(G.to_dev(zu), zu, np.zeros((2, p.N), np.int64), np.zeros((2, p.N), np.uint64))
+    assert e.value.status == -1

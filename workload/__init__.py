@@ -96,13 +96,22 @@ CONFIGS = {
                         glwe_sigma_log2=13, lut=("exp", -8.0, 0.0),
                         msg=("normal", 2.0, -8.0, 0.0), batch=1024, seed=5,
                         batches=(1, 64, 1024, 16384, 65536)),
+    # Encrypted segmented lookup on a small ring (two traces multiply the
+    # result by N^2, so the noise of a blind rotation must stay well below
+    # 2^63 / N^2): n=64, N=512, PBS 2^8 x 6, KS 2^4 x 8, 1/x on [0.1, 2.0]
+    # with the paper's two segments and four intervals per segment.
+    "lookup_small": Params("lookup_small", n=64, k=1, N=512, pbs_base_log=8, pbs_level=6,
+                           ks_base_log=4, ks_level=8, msg_bits=2, lwe_sigma_log2=30,
+                           glwe_sigma_log2=13, lut=("reciprocal", 0.1, 2.0),
+                           msg=("uniform",), batch=8, seed=6),
 }
 
 # purposes of independent random streams
 _PURPOSE = {
     "lwe_key": 1, "glwe_key": 2, "bsk_mask": 3, "bsk_noise": 4, "ksk_mask": 5,
     "ksk_noise": 6, "ct_mask": 7, "ct_noise": 8, "messages": 9, "uniform_keys": 10,
-    "uniform_cts": 11, "sample": 12,
+    "uniform_cts": 11, "sample": 12, "trace_mask": 13, "trace_noise": 14, "glwe_mask": 15,
+    "glwe_noise": 16, "inputs": 17,
 }
 
 
@@ -161,7 +170,7 @@ def lut_codes(params: Params) -> np.ndarray:
     if params.lut[0] == "square_mod":
         return np.array([(m * m) % size for m in range(size)], dtype=np.int64)
     kind, lo, hi = params.lut
-    f = {"gelu": _gelu, "silu": _silu, "exp": math.exp}[kind]
+    f = {"gelu": _gelu, "silu": _silu, "exp": math.exp, "reciprocal": lambda x: 1.0 / x}[kind]
     ys = [f(x) for x in bin_midpoints(lo, hi, size)]
     y_lo, y_hi = min(ys), max(ys)
     codes = [min(max(math.floor((y - y_lo) / (y_hi - y_lo) * (size - 1) + 0.5), 0), size - 1) for y in ys]

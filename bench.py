@@ -8,6 +8,11 @@ PBS base 2^23 x 1, KS base 2^3 x 5) on a batch of 4096 ciphertexts with a
 
 Prints one JSON line (rank 0).  `--impl reference` times the CPU oracle on
 the host cores instead (the reference arm: a deliberately plain program).
+
+`--path lookup` measures the encrypted segmented lookup instead (the
+lookup protocol's Steps 2 and 3 composed from plaintext products, blind
+rotations of GLWE test polynomials, a key switch and RLWE traces) on the
+same ring, four segments, one line of its own.
 """
 
 from __future__ import annotations
@@ -58,6 +63,36 @@ def int_ops_per_pbs(p):
                 + k1 * N * 10 * P + k1 * N * l * 6 + k1 * N * 4)
     ks = p.kN * p.ks_level * (p.n + 1) * 3 + p.kN * p.ks_level * 6
     return per_cmux * p.n, ks
+
+
+def _ntt_ops(N: int) -> int:
+    return (N // 2) * int(math.log2(N)) * 8
+
+
+def _primes_for(bits: float) -> int:
+    return math.ceil(bits / 31)
+
+
+def int_ops_key_switch_step(N: int, base_log: int, rows: int, outs: int = 2) -> int:
+    """One GLWE key switch (trace step) or plaintext product: `rows` digit
+    polynomials times `outs` key components, same convention as above."""
+    P = _primes_for(63 + (base_log - 1) + math.log2(rows * N) + 1)
+    return ((rows + outs) * P * _ntt_ops(N) + rows * outs * P * N * 6 + outs * N * 10 * P
+            + N * rows * 6 + outs * N * 4)
+
+
+def int_ops_per_lookup(p, n_seg: int, t_base_log: int, t_level: int) -> dict:
+    """Per encrypted lookup: n_seg + 2 blind rotations, one key switch,
+    n_seg + 1 traces (log2 N key-switch steps each), n_seg + 2 plaintext
+    products (exact 16 x 4 gadget on both components: 8 rows; per output
+    only 4 are nonzero, which bounds the primes)."""
+    br, ks = int_ops_per_pbs(p)
+    logN = int(math.log2(p.N))
+    tr = logN * int_ops_key_switch_step(p.N, t_base_log, t_level)
+    P = _primes_for(63 + 15 + math.log2(4 * p.N) + 1)
+    pm = (8 + 2) * P * _ntt_ops(p.N) + 8 * 2 * P * p.N * 6 + 2 * p.N * 10 * P + 2 * p.N * 4 * 6 + 2 * p.N * 4
+    return {"blind_rotation": (n_seg + 2) * br, "key_switch": ks, "trace": (n_seg + 1) * tr,
+            "plaintext_mul": (n_seg + 2) * pm, "monomial": n_seg * 2 * p.N * 2}
 
 
 TRAFFIC_SUMMARY = os.path.join(ROOT, "profiles", "blind_rotate_standard_b4096_dram.txt")
@@ -189,6 +224,92 @@ def run_reference(args, p, batch):
     print(json.dumps(line), flush=True)
 
 
+# ---------------------------------------------------------------------------- lookup path
+
+LOOKUP_METRIC = "encrypted segmented lookups/sec (lookup protocol Steps 2-3, 4 segments) on 1 GB300"
+LOOKUP_SEGMENTS, LOOKUP_TRACE = 4, (16, 4)
+
+
+def run_lookup(args, p, batch, torch, dev, R, clock_sampler):
+    """Throughput of rosetta_segmented_lookup_batch on `batch` ciphertexts,
+    plus each component entry point timed alone on the same batch."""
+    n_seg = LOOKUP_SEGMENTS
+    tb, tl = LOOKUP_TRACE
+    g = np.random.default_rng(p.seed)
+
+    def d(a):
+        return torch.from_numpy(np.ascontiguousarray(a).view(np.int64)).to(dev)
+
+    bsk, ksk = W.uniform_keys(p)
+    ctx = R.Context(p, device=dev.index or 0)
+    ctx.upload_bsk(d(bsk))
+    ctx.upload_ksk(d(ksk))
+    del bsk, ksk
+    steps = int(math.log2(p.N))
+    ctx.upload_trace_keys(d(W.uniform_u64((steps, tl, 2, p.N), W.rng(p.seed, "sample", 300))), tb, tl)
+    tables = (g.integers(-2**40, 2**40, size=p.N, dtype=np.int64), W.uniform_u64((p.N,), W.rng(p.seed, "sample", 301)),
+              g.integers(-2**40, 2**40, size=(n_seg, p.N), dtype=np.int64),
+              W.uniform_u64((n_seg, p.N), W.rng(p.seed, "sample", 302)))
+    ctx.upload_lookup_table(*tables)
+    glwe = d(W.uniform_u64((batch, 2, p.N), W.rng(p.seed, "sample", 303)))
+    lwe = d(W.uniform_ciphertexts(p, batch, sub=7))
+    out = torch.empty((batch, 2, p.N), dtype=torch.int64, device=dev)
+    tmp = torch.empty((batch, 2, p.N), dtype=torch.int64, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.int32, device=dev)
+    for _ in range(max(3, args.warmup)):
+        ctx.segmented_lookup_batch(glwe, lwe, out, stream)
+    ctx.sync_status(stream)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    torch.cuda.synchronize(dev)
+    with clock_sampler(dev.index or 0) as clk:
+        for s in range(args.steps):
+            flush.zero_()
+            ev[s][0].record(stream)
+            ctx.segmented_lookup_batch(glwe, lwe, out, stream)
+            ev[s][1].record(stream)
+        torch.cuda.synchronize(dev)
+    ctx.sync_status(stream)
+    total_ms = sum(a.elapsed_time(b) for a, b in ev)
+    value = batch * args.steps / (total_ms / 1e3)
+
+    def timed(fn, reps=3):
+        e = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
+        for i in range(reps):
+            flush.zero_()
+            e[i][0].record(stream)
+            fn()
+            e[i][1].record(stream)
+        ctx.sync_status(stream)
+        return statistics.mean(a.elapsed_time(b) for a, b in e)
+
+    br_ms = timed(lambda: ctx.blind_rotate_glwe_batch(lwe, glwe, tmp, stream))
+    tr_ms = timed(lambda: ctx.trace_batch(glwe, tmp, stream))
+    ops = int_ops_per_lookup(p, n_seg, tb, tl)
+    br_ops = int_ops_per_pbs(p)[0]
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    sm_max = peaks().get("sm_max_mhz", 2070.0)
+    alu_peak = sms * 128 * sm_max * 1e6 / 1e12
+    achieved = br_ops * batch / (br_ms / 1e3) / 1e12
+    path_achieved = sum(ops.values()) * batch * args.steps / (total_ms / 1e3) / 1e12
+    line = {
+        "metric": LOOKUP_METRIC, "value": value, "unit": "lookups/s", "n_gpus": 1, "steps": args.steps,
+        "warmup": max(3, args.warmup), "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "u64", "data": "synthetic",
+        "config": {"workload": f"segmented lookup, {n_seg} segments, ring of {describe(p, batch)}, "
+                               f"trace gadget 2^{tb} x {tl}", "batch": batch,
+                   "l2": "flushed between steps (256 MB write)", "keys": "uniform words, resident"},
+        "roofline": {"bound": "alu", "kernel": "blind_rotate_kernel (GLWE test polynomials)", "achieved": achieved,
+                     "peak": alu_peak, "unit": "Tops/s (int32)", "frac": achieved / alu_peak, "traffic": None,
+                     "kernel_ms": br_ms, "trace_ms": tr_ms,
+                     "path_ops_per_lookup": ops, "path_achieved": path_achieved,
+                     "path_frac": path_achieved / alu_peak},
+        "gpu_launches": (4 * n_seg + 6) * args.steps,
+        "clocks": clk.summary(),
+    }
+    print(json.dumps(line), flush=True)
+
+
 # ---------------------------------------------------------------------------- GPU arm
 
 def main():
@@ -201,11 +322,19 @@ def main():
     ap.add_argument("--batch", type=int, default=0, help="override the workload's batch")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-sample", type=int, default=0, help="oracle sample size (default: host cores)")
+    ap.add_argument("--path", default="pbs", choices=["pbs", "lookup"])
     args = ap.parse_args()
     p = W.CONFIGS[args.config]
     batch = args.batch or p.batch
     if args.impl == "reference":
         return run_reference(args, p, batch)
+    if args.path == "lookup":
+        import torch
+        import paper_2609_16915_gb300 as R
+        R.load()
+        dev = torch.device("cuda", 0)
+        torch.cuda.set_device(dev)
+        return run_lookup(args, p, args.batch or 1024, torch, dev, R, ClockSampler)
 
     import torch
     world = int(os.environ.get("WORLD_SIZE", "1"))

@@ -10,7 +10,7 @@
 // The external product decomposes each coefficient of the rotated difference
 // into signed digits and forms sum_r D_r * BSK_i[r][c] in Z_{2^64}[X]/(X^N+1).
 // Those products are computed exactly: the integer value of every output
-// coefficient is below M/2 with M the product of four 29-bit NTT primes, so
+// coefficient is below M/2 with M the product of four 28-bit NTT primes, so
 // four negacyclic NTTs, a pointwise multiply-accumulate per prime and an
 // explicit CRT (X = sum_q y_q M/p_q - round(sum_q y_q/p_q) M, evaluated mod
 // 2^64) give the same words as the schoolbook product.
@@ -63,7 +63,9 @@ struct BrShape {
   static constexpr int MIN_CTAS = (LOGN <= 11) ? 4 : (LOGN == 12 ? 2 : 1);
 };
 
-template <int LOGN, bool DIG16>
+// LEV > 0 fixes the gadget level count at compile time (the common sets:
+// straight-line digit and key loops); LEV = 0 reads it from the arguments.
+template <int LOGN, bool DIG16, int LEV>
 __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) blind_rotate_kernel(const BrArgs a) {
   using B = BrShape<LOGN>;
   using S = NttShape<LOGN, B::E>;
@@ -83,7 +85,8 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
   uint32_t *res = reinterpret_cast<uint32_t *>(acc + 2 * Q);     // [4 primes][2][Q]
   uint32_t *xb = res + kPrimes * 2 * Q;                          // [XBUF][XB_WORDS]
   DigT *dig = reinterpret_cast<DigT *>(xb + B::XBUF * S::XB_WORDS);  // [2l][Q]
-  uint16_t *atil = reinterpret_cast<uint16_t *>(dig + 2 * a.level * Q);  // [n+1]
+  const uint32_t level = LEV > 0 ? static_cast<uint32_t>(LEV) : a.level;
+  uint16_t *atil = reinterpret_cast<uint16_t *>(dig + 2 * level * Q);  // [n+1]
 
   const uint32_t p = a.cc.pr[rank].p;
   const uint32_t p_inv = a.cc.pr[rank].p_inv;
@@ -143,8 +146,8 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
   // 32-bit shared-memory addresses; mapa turns them into the same location
   // in another CTA of the cluster
   const uint32_t acc_s = smem_addr(acc), dig_s = smem_addr(dig), res_s = smem_addr(res);
-  const uint32_t L2 = 2 * a.level;
-  const uint32_t bits = a.base_log * a.level;
+  const uint32_t L2 = 2 * level;
+  const uint32_t bits = a.base_log * level;
   const uint64_t Bmask = (1ull << a.base_log) - 1;
   const uint64_t Bhalf = 1ull << (a.base_log - 1);
   const uint64_t round_add = bits >= 64 ? 0 : (1ull << (63 - bits));
@@ -172,7 +175,8 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
       const bool neg = ((j + TWO_N - at) & (TWO_N - 1)) >= N;
       const uint64_t diff = (neg ? 0ull - v[m] : v[m]) - acc[c * Q + jl];
       uint64_t cv = bits >= 64 ? diff : (diff + round_add) >> round_sh;
-      for (int l = static_cast<int>(a.level) - 1; l >= 0; --l) {
+#pragma unroll
+      for (int l = static_cast<int>(level) - 1; l >= 0; --l) {
         const uint64_t d = cv & Bmask;
         cv >>= a.base_log;
         int32_t ds = static_cast<int32_t>(d);
@@ -180,7 +184,7 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
           ds -= static_cast<int32_t>(Bmask + 1);
           cv += 1;
         }
-        dig[(c * a.level + l) * Q + jl] = static_cast<DigT>(ds);
+        dig[(c * level + l) * Q + jl] = static_cast<DigT>(ds);
       }
     }
     cluster.sync();
@@ -188,6 +192,7 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
     // ---- phase 2: transforms and pointwise products for prime `rank` ----
     uint32_t oh[2][E];
     const uint32_t *gbase = a.bsk + (static_cast<size_t>(i) * kPrimes + rank) * (static_cast<size_t>(L2) * 2 * N);
+#pragma unroll 1
     for (uint32_t r0 = 0; r0 < L2; r0 += 2) {
       // first-pass slot q of thread tau is coefficient tau + q N/E, owned by
       // CTA q / QE at local index tau + (q % QE) T
@@ -217,12 +222,12 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
 #pragma unroll
           for (int pp = 0; pp < 2; ++pp)
 #pragma unroll
-            for (int e = 0; e < E; ++e) x[pp][e] = cond_sub(x[pp][e], 4 * p);  // < 8p -> < 4p
+            for (int e = 0; e < E; ++e) x[pp][e] = cond_sub(x[pp][e], 8 * p);  // < 16p -> < 8p
         }
 #pragma unroll
         for (int e = 0; e < E; ++e) {
-          // forward outputs < 4p, BSK words < p in Montgomery form: the pair
-          // sum stays below p * 2^32
+          // forward outputs < 8p, BSK words < p in Montgomery form: the pair
+          // sum stays below 16 p^2 < p * 2^32
           const uint64_t prod = static_cast<uint64_t>(x[0][e]) * ga[e] + static_cast<uint64_t>(x[1][e]) * gb[e];
           const uint32_t rr = redc(prod, p, p_inv);  // (0, 2p)
           oh[c][e] = (r0 == 0) ? rr : cond_sub(oh[c][e] + rr, 4 * p);
@@ -250,9 +255,9 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
       for (int pq = 0; pq < kPrimes; ++pq) {
         const uint32_t y = res[(pq * 2 + c) * Q + jl];
         s += static_cast<uint64_t>(y) * a.cc.pr[pq].Mp_mod64;
-        frac += __umulhi(y, a.cc.pr[pq].F);  // y / p in units of 2^-28
+        frac += __umulhi(y, a.cc.pr[pq].F);  // y / p in units of 2^-27
       }
-      const uint32_t u = (frac + (1u << 27)) >> 28;  // round(sum y_q / p_q)
+      const uint32_t u = (frac + (1u << 26)) >> 27;  // round(sum y_q / p_q)
       acc[c * Q + jl] += s - static_cast<uint64_t>(u) * a.cc.M_mod64;
     }
     cluster.sync();
@@ -292,9 +297,9 @@ size_t br_smem_bytes(uint32_t logN, uint32_t level, uint32_t n, bool dig16) {
   return (b + 15) & ~size_t(15);
 }
 
-template <int LOGN, bool DIG16>
+template <int LOGN, bool DIG16, int LEV>
 static cudaError_t launch_br_t(const BrArgs &a, cudaStream_t s) {
-  auto kern = blind_rotate_kernel<LOGN, DIG16>;
+  auto kern = blind_rotate_kernel<LOGN, DIG16, LEV>;
   const size_t smem = br_smem_bytes(LOGN, a.level, a.n, DIG16);
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e == cudaSuccess)
@@ -315,10 +320,23 @@ static cudaError_t launch_br_t(const BrArgs &a, cudaStream_t s) {
   return cudaLaunchKernelEx(&cfg, kern, a);
 }
 
+template <int LOGN, bool DIG16>
+static cudaError_t launch_br_lev(const BrArgs &a, cudaStream_t s) {
+  if constexpr (LOGN >= 11) {
+    // (a fixed count of 2 measured slower at N = 4096 than the runtime loop)
+    switch (a.level) {
+      case 1: return launch_br_t<LOGN, DIG16, 1>(a, s);
+      case 3: return launch_br_t<LOGN, DIG16, 3>(a, s);
+      default: break;
+    }
+  }
+  return launch_br_t<LOGN, DIG16, 0>(a, s);
+}
+
 cudaError_t launch_blind_rotate(const BrArgs &a, uint32_t logN, bool dig16, cudaStream_t s) {
 #define ROSETTA_BR_CASE(L)                                                        \
   case L:                                                                         \
-    return dig16 ? launch_br_t<L, true>(a, s) : launch_br_t<L, false>(a, s);
+    return dig16 ? launch_br_lev<L, true>(a, s) : launch_br_lev<L, false>(a, s);
   switch (logN) {
     ROSETTA_BR_CASE(8)
     ROSETTA_BR_CASE(9)

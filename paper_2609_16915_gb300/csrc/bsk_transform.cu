@@ -49,7 +49,7 @@ __global__ void __launch_bounds__((1 << LOGN) / 8)
   uint32_t *dst = out + (((static_cast<size_t>(i) * kPrimes + q) * rows + r) * 2 + c) * N + 8 * tau;
 #pragma unroll
   for (int e = 0; e < 8; ++e) {
-    uint32_t v = cond_sub(cond_sub(cond_sub(x[0][e], 4 * p), 2 * p), p);  // < 8p -> < p
+    uint32_t v = cond_sub(cond_sub(cond_sub(cond_sub(x[0][e], 8 * p), 4 * p), 2 * p), p);  // < 16p -> < p
     v = cond_sub(shoup_mul(v, pc.r_mont, pc.r_mont_s, p), p);
     dst[e] = v;
   }

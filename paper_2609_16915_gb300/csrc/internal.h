@@ -6,20 +6,20 @@
 
 namespace rosetta {
 
-// Four NTT primes p = c * 2^14 + 1 in (2^28, 2^29): 2N | p - 1 for every
-// N <= 8192, 8p < 2^32 leaves room for lazily reduced residues, and their
-// product M > 2^115 exceeds twice the largest exact integer value of an
+// Four NTT primes p = c * 2^14 + 1 in (2^27, 2^28): 2N | p - 1 for every
+// N <= 8192, 16p < 2^32 leaves room for lazily reduced residues, and their
+// product M > 2^111.99 exceeds twice the largest exact integer value of an
 // external-product coefficient, (k+1) l N 2^(beta-1) 2^63, for every
 // parameter set the library accepts (checked at context creation).
 constexpr int kPrimes = 4;
-constexpr uint32_t kPrimeList[kPrimes] = {536690689u, 536641537u, 536608769u, 536543233u};
+constexpr uint32_t kPrimeList[kPrimes] = {268369921u, 268271617u, 268238849u, 268189697u};
 
 struct PrimeConsts {
   uint32_t p;
   uint32_t p_inv;     // p^{-1} mod 2^32 (Montgomery reduction)
   uint32_t crt_c;     // N^{-1} * (M/p)^{-1} mod p
   uint32_t crt_cs;    // Shoup companion of crt_c
-  uint32_t F;         // floor(2^60 / p): fixed-point 1/p for the CRT quotient
+  uint32_t F;         // floor(2^59 / p): fixed-point 1/p for the CRT quotient
   uint32_t r_mont;    // 2^32 mod p
   uint32_t r_mont_s;  // Shoup companion of r_mont
   uint32_t pad_;

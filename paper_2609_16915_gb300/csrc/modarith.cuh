@@ -1,4 +1,4 @@
-// Word-level modular arithmetic for the NTT primes (p < 2^29, so 8p < 2^32
+// Word-level modular arithmetic for the NTT primes (p < 2^28, so 16p < 2^32
 // and lazily reduced residues up to 8p still fit a 32-bit register).
 //
 // Residues are kept "lazy": a value congruent to the residue but possibly a

@@ -18,7 +18,7 @@
 // inverse pass needs, so a pointwise product between the two transforms
 // needs no exchange.
 //
-// Lazy ranges: forward input < 2p, output < 8p; inverse input < 4p, output
+// Lazy ranges: forward input < 2p, output < 16p; inverse input < 4p, output
 // < 4p.  See the butterflies for the per-stage invariants.
 #pragma once
 #include <stdint.h>
@@ -68,19 +68,21 @@ __device__ __forceinline__ uint32_t slot_index(uint32_t tau, int e) {
 
 // Forward (Cooley-Tukey) butterfly X' = X + wY, Y' = X - wY with t = wY in
 // [0, 2p).  Without correction: inputs < a p give outputs < (a+2) p.  With
-// correction X is first brought below 4p (valid for X < 8p).
+// correction X is first brought below 8p (valid for X < 16p), so the outputs
+// are below 10p whatever Y was.
 template <bool CORR>
 __device__ __forceinline__ void ct_bfly(uint32_t &X, uint32_t &Y, uint2 w, uint32_t p, uint32_t two_p,
-                                        uint32_t four_p) {
-  if (CORR) X = cond_sub(X, four_p);
+                                        uint32_t eight_p) {
+  if (CORR) X = cond_sub(X, eight_p);
   const uint32_t t = shoup_mul(Y, w.x, w.y, p);
   Y = X - t + two_p;
   X = X + t;
 }
 
-// Stage s of the forward transform corrects X when s >= 3 and s is odd:
-// bounds run 2p -> 4p -> 6p -> 8p, then alternate 6p (corrected) and 8p.
-__host__ __device__ constexpr bool fwd_stage_corrects(int s) { return s >= 3 && ((s - 3) % 2 == 0); }
+// Stage s of the forward transform corrects X when s = 7, 11, 15, ...: the
+// bounds run 2p -> 4p -> .. -> 16p after stage 6, then 10p (corrected),
+// 12p, 14p, 16p, 10p (corrected), ...; 16p < 2^32.
+__host__ __device__ constexpr bool fwd_stage_corrects(int s) { return s >= 7 && ((s - 7) % 4 == 0); }
 
 // Inverse (Gentleman-Sande) butterfly with inverse twiddle -w:
 // X' = X + Y, Y' = (X - Y)(-w) = (Y - X + 4p) w.  Inputs < 4p give X' < 8p,
@@ -124,7 +126,7 @@ __device__ __forceinline__ void load_twiddles(const uint2 *__restrict__ tw, uint
 
 template <int LOGN, int E, int NP, int S0, int H, int U>
 __device__ __forceinline__ void fwd_stage(uint32_t (&x)[NP][E], const uint2 *__restrict__ tw, uint32_t tau,
-                                          uint32_t p, uint32_t two_p, uint32_t four_p) {
+                                          uint32_t p, uint32_t two_p, uint32_t eight_p) {
   constexpr uint32_t N = 1u << LOGN;
   constexpr uint32_t SIG = N >> (S0 + H);
   constexpr int NB = E >> H;
@@ -144,7 +146,7 @@ __device__ __forceinline__ void fwd_stage(uint32_t (&x)[NP][E], const uint2 *__r
 #pragma unroll
         for (int k = 0; k < NP; ++k)
           ct_bfly<CORR>(x[k][b * (1 << H) + q], x[k][b * (1 << H) + q + HALF], w[(b << U) + (q >> (H - U))], p, two_p,
-                        four_p);
+                        eight_p);
       }
   } else {
 #pragma unroll
@@ -156,7 +158,7 @@ __device__ __forceinline__ void fwd_stage(uint32_t (&x)[NP][E], const uint2 *__r
         const uint2 w = tw[(1u << S) + (g << U) + (q >> (H - U))];
 #pragma unroll
         for (int k = 0; k < NP; ++k)
-          ct_bfly<CORR>(x[k][b * (1 << H) + q], x[k][b * (1 << H) + q + HALF], w, p, two_p, four_p);
+          ct_bfly<CORR>(x[k][b * (1 << H) + q], x[k][b * (1 << H) + q + HALF], w, p, two_p, eight_p);
       }
     }
   }
@@ -205,9 +207,9 @@ __device__ __forceinline__ void inv_stage(uint32_t (&x)[NP][E], const uint2 *__r
 
 template <int LOGN, int E, int NP, int S0, int H, int U = 0>
 __device__ __forceinline__ void fwd_pass(uint32_t (&x)[NP][E], const uint2 *tw, uint32_t tau, uint32_t p,
-                                         uint32_t two_p, uint32_t four_p) {
-  fwd_stage<LOGN, E, NP, S0, H, U>(x, tw, tau, p, two_p, four_p);
-  if constexpr (U + 1 < H) fwd_pass<LOGN, E, NP, S0, H, U + 1>(x, tw, tau, p, two_p, four_p);
+                                         uint32_t two_p, uint32_t eight_p) {
+  fwd_stage<LOGN, E, NP, S0, H, U>(x, tw, tau, p, two_p, eight_p);
+  if constexpr (U + 1 < H) fwd_pass<LOGN, E, NP, S0, H, U + 1>(x, tw, tau, p, two_p, eight_p);
 }
 
 template <int LOGN, int E, int NP, int S0, int H, int U = H - 1>
@@ -332,7 +334,7 @@ __device__ __forceinline__ void ntt_forward(uint32_t (&x)[NP][E], const uint2 *t
   using S = NttShape<LOGN, E>;
   constexpr int S0 = S::RAD * PASS;
   constexpr int H = S::template h<PASS>();
-  fwd_pass<LOGN, E, NP, S0, H>(x, tw, tau, p, 2 * p, 4 * p);
+  fwd_pass<LOGN, E, NP, S0, H>(x, tw, tau, p, 2 * p, 8 * p);
   if constexpr (PASS + 1 < S::NPASS) {
     exchange<LOGN, E, NP, XBUF, S0, H, S0 + S::RAD, S::template h<PASS + 1>()>(x, xb, tau);
     ntt_forward<LOGN, E, NP, XBUF, PASS + 1>(x, tw, xb, tau, p);

@@ -62,8 +62,8 @@ int check_params(const rosetta_params &p) {
   if (p.ks_base_log < 1 || p.ks_base_log > 16 || p.ks_level < 1 || p.ks_base_log * p.ks_level > 64)
     return ROSETTA_ERR_UNSUPPORTED_PARAMS;
   if (p.msg_bits < 1 || p.msg_bits > 62 || (p.poly_size >> p.msg_bits) < 2) return ROSETTA_ERR_UNSUPPORTED_PARAMS;
-  // exact CRT: the product of the four primes (> 2^115) must exceed twice the bound
-  if (ext_product_bits(p) + 1.0 > 115.0) return ROSETTA_ERR_UNSUPPORTED_PARAMS;
+  // exact CRT: the product of the four primes (> 2^111.99) must exceed twice the bound
+  if (ext_product_bits(p) + 1.0 > 111.0) return ROSETTA_ERR_UNSUPPORTED_PARAMS;
   return ROSETTA_OK;
 }
 
@@ -466,7 +466,7 @@ int rosetta_upload_trace_keys(rosetta_ctx *c, const uint64_t *keys, size_t n_wor
   {
     int e = 0;
     while ((1ull << e) < (uint64_t)level * p.poly_size) ++e;
-    if (63 + (base_log - 1) + e + 1 > 115) return ROSETTA_ERR_UNSUPPORTED_PARAMS;
+    if (63 + (base_log - 1) + e + 1 > 111) return ROSETTA_ERR_UNSUPPORTED_PARAMS;
   }
   int max_smem = 0;
   cudaDeviceGetAttribute(&max_smem, cudaDevAttrMaxSharedMemoryPerBlockOptin, c->device);

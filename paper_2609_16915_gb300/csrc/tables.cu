@@ -67,7 +67,7 @@ bool build_tables(uint32_t logN, uint2 *tw_host, CrtConsts *cc) {
   cc->M_mod64 = static_cast<uint64_t>(M);
   for (int q = 0; q < kPrimes; ++q) {
     const uint32_t p = kPrimeList[q];
-    if (!is_prime(p) || (p - 1) % (2 * N) != 0 || p >= (1u << 29) || p <= (1u << 28)) return false;
+    if (!is_prime(p) || (p - 1) % (2 * N) != 0 || p >= (1u << 28) || p <= (1u << 27)) return false;
     const uint32_t g = generator(p);
     if (!g) return false;
     const uint32_t psi = powmod(g, (p - 1) / (2 * N), p);  // primitive 2N-th root of unity
@@ -87,7 +87,7 @@ bool build_tables(uint32_t logN, uint2 *tw_host, CrtConsts *cc) {
     const uint32_t N_inv = powmod(N, p - 2, p);
     pc.crt_c = static_cast<uint32_t>(static_cast<uint64_t>(Mq_inv) * N_inv % p);
     pc.crt_cs = shoup(pc.crt_c, p);
-    pc.F = static_cast<uint32_t>((static_cast<u128>(1) << 60) / p);
+    pc.F = static_cast<uint32_t>((static_cast<u128>(1) << 59) / p);
     pc.r_mont = static_cast<uint32_t>((static_cast<uint64_t>(1) << 32) % p);
     pc.r_mont_s = shoup(pc.r_mont, p);
     pc.pad_ = 0;

@@ -163,7 +163,7 @@ __global__ void __launch_bounds__(TrShape<LOGN>::T) trace_kernel(const TraceArgs
 #pragma unroll
           for (int pp = 0; pp < 2; ++pp)
 #pragma unroll
-            for (int e = 0; e < E; ++e) x[pp][e] = cond_sub(x[pp][e], 4 * p);
+            for (int e = 0; e < E; ++e) x[pp][e] = cond_sub(x[pp][e], 8 * p);
         }
 #pragma unroll
         for (int e = 0; e < E; ++e) {
@@ -196,7 +196,7 @@ __global__ void __launch_bounds__(TrShape<LOGN>::T) trace_kernel(const TraceArgs
         sum += static_cast<uint64_t>(y) * a.cc.pr[pq].Mp_mod64;
         frac += __umulhi(y, a.cc.pr[pq].F);
       }
-      const uint32_t u = (frac + (1u << 27)) >> 28;
+      const uint32_t u = (frac + (1u << 26)) >> 27;
       const uint64_t X = sum - static_cast<uint64_t>(u) * a.cc.M_mod64;
       if (PTMUL)
         acc[c * Q + jl] = X + ((c == 1 && a.plain_add) ? a.plain_add[rank * Q + jl] : 0ull);

@@ -95,6 +95,28 @@ def int_ops_per_lookup(p, n_seg: int, t_base_log: int, t_level: int) -> dict:
             "plaintext_mul": (n_seg + 2) * pm, "monomial": n_seg * 2 * p.N * 2}
 
 
+def ks_tensor_limbs(p, batch) -> int:
+    """Limbs per key word of the tensor-core key switch the library takes for
+    this batch (8 or 16), or 0 when it takes the CUDA-core kernel: batches of
+    256 and more, digits that bf16 holds, fp32 sums below 2^24."""
+    K = p.kN * p.ks_level
+    if batch < 256 or p.ks_base_log > 8 or K % 64:
+        return 0
+    for limbs in (8, 16):
+        if 2 ** (p.ks_base_log - 1) * (2 ** (64 // limbs) - 1) * K < 2 ** 24:
+            return limbs
+    return 0
+
+
+def ks_tensor_flops(p, batch, limbs) -> float:
+    """Dense bf16 flops of the tensor-core key switch as launched: 128-row by
+    256-column output tiles over K = kN l."""
+    K = p.kN * p.ks_level
+    rows = -(-batch // 128) * 128
+    cols = -(-(p.n + 1) * limbs // 256) * 256
+    return 2.0 * rows * K * cols
+
+
 TRAFFIC_SUMMARY = os.path.join(ROOT, "profiles", "blind_rotate_standard_b4096_dram.txt")
 
 
@@ -433,6 +455,17 @@ def main():
     br_ops, ks_ops = int_ops_per_pbs(p)
     achieved = br_ops * batch / (br_ms / 1e3) / 1e12
     pbs_roof = alu_peak * 1e12 / (br_ops + ks_ops)
+    limbs = ks_tensor_limbs(p, batch)
+    if limbs:
+        ks_tf = ks_tensor_flops(p, batch, limbs) / (ks_ms / 1e3) / 1e12
+        bf16_peak = pk.get("bf16_tflops", 1900.0)
+        ks_roof = {"bound": "tensor", "kernel": "ks_digits_kernel + ks_tc_kernel (bf16 tcgen05)",
+                   "achieved": ks_tf, "peak": bf16_peak, "unit": "TFLOP/s", "frac": ks_tf / bf16_peak,
+                   "limbs": limbs, "peak_basis": "bf16_tflops of MEASURED_PEAKS.json (burst)"}
+    else:
+        ks_roof = {"bound": "alu", "kernel": "keyswitch_kernel", "achieved": ks_ops * batch / (ks_ms / 1e3) / 1e12,
+                   "peak": alu_peak, "unit": "Tops/s (int32)"}
+        ks_roof["frac"] = ks_roof["achieved"] / alu_peak
 
     if rank != 0:
         if dist:
@@ -447,11 +480,11 @@ def main():
         "roofline": {"bound": "alu", "kernel": "blind_rotate_kernel", "achieved": achieved, "peak": alu_peak,
                      "unit": "Tops/s (int32)", "frac": achieved / alu_peak, "traffic": measured_traffic(p, batch),
                      "peak_basis": f"{sms} SMs x 128 int32 lanes x {sm_max:.0f} MHz (sm_max_mhz of MEASURED_PEAKS.json)",
-                     "kernel_ms": br_ms, "keyswitch_ms": ks_ms,
+                     "kernel_ms": br_ms, "keyswitch_ms": ks_ms, "keyswitch": ks_roof,
                      "pbs_roof": pbs_roof, "pbs_frac_of_roof": value / world / pbs_roof},
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": batch * (p.n + 1) * 8 + lut.numel() * 8,
                 "d2h_bytes_per_step": batch * (p.n + 1) * 8},
-        "gpu_launches": 2 * args.steps,
+        "gpu_launches": (3 if limbs else 2) * args.steps,
         "clocks": clk.summary(),
         "wall_s_timed": wall,
     }

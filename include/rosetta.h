@@ -124,7 +124,13 @@ int rosetta_blind_rotate_extract_batch(rosetta_ctx *ctx, const uint64_t *lwe_in,
  * [batch][kN+1], to dimension n, lwe_out [batch][n+1]:
  *   out = (0, .., 0, b') - sum_i sum_lev d_{i,lev}(a'_i) * KSK[i][lev]
  * with d the signed base-2^beta_ks digits of a'_i rounded to its top
- * beta_ks*l_ks bits.  Needs the KSK. */
+ * beta_ks*l_ks bits.  Needs the KSK.  From 256 ciphertexts on, where the
+ * parameters allow exact fp32 sums (beta_ks <= 8 and
+ * 2^(beta_ks-1) (2^(64/limbs)-1) kN l_ks < 2^24 for 8 or 16 limbs per key
+ * word), the product runs on the tensor cores with a digit scratch of
+ * batch (kN l_ks) bf16 words owned by the context; the words are the same
+ * either way.  A bounded wait inside that kernel that gives up is reported
+ * as TIMEOUT by rosetta_sync_status. */
 int rosetta_keyswitch_batch(rosetta_ctx *ctx, const uint64_t *lwe_big_in, uint32_t batch,
                             uint64_t *lwe_out, void *stream);
 
@@ -247,8 +253,9 @@ int rosetta_pbs_batch_noalloc(rosetta_ctx *ctx, const uint64_t *lwe_in, uint32_t
                               const uint64_t *lut, uint64_t *lwe_out, void *stream);
 
 /* Wait for all work on `stream` and report any deferred execution error
- * (CUDA, TIMEOUT, or INVALID_ARG for an out-of-range LUT index seen by
- * rosetta_pbs_batch_multi_lut; that flag is cleared once reported).  Returns
+ * (CUDA; TIMEOUT when a bounded wait of the tensor-core key switch gave up;
+ * INVALID_ARG for an out-of-range LUT index seen by
+ * rosetta_pbs_batch_multi_lut; the flag is cleared once reported).  Returns
  * OK when the stream finished cleanly. */
 int rosetta_sync_status(rosetta_ctx *ctx, void *stream);
 

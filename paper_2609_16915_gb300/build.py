@@ -16,7 +16,8 @@ CSRC = os.path.join(HERE, "csrc")
 ROOT = os.path.dirname(HERE)
 LIB = os.path.join(HERE, "librosetta.so")
 BUILD_DIR = os.path.join(ROOT, "_build")
-SOURCES = ["tables.cu", "bsk_transform.cu", "blind_rotate.cu", "keyswitch.cu", "rosetta_api.cu", "pbs_noalloc.cu", "trace.cu"]
+SOURCES = ["tables.cu", "bsk_transform.cu", "blind_rotate.cu", "keyswitch.cu", "keyswitch_tc.cu", "rosetta_api.cu",
+           "pbs_noalloc.cu", "trace.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

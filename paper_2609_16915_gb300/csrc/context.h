@@ -18,6 +18,10 @@ struct rosetta_ctx {
   uint32_t *d_bsk = nullptr;      // transform domain
   uint64_t *d_ksk = nullptr;      // raw [kN][l_ks][n+1]
   uint64_t *d_corr = nullptr;     // [n+1]
+  uint16_t *d_ks_b = nullptr;     // key limb tiles for the tensor-core key switch (null: not exact)
+  uint32_t ks_limbs = 0;
+  uint64_t *d_ks_a = nullptr;     // digit tiles (scratch), as 64-bit words
+  size_t ks_a_cap = 0;
   bool have_bsk = false, have_ksk = false;
   // scratch and staging, sized in ciphertexts
   uint64_t *d_big = nullptr;      // extracted ciphertexts [batch][kN+1]

@@ -53,6 +53,16 @@ struct KsArgs {
   uint32_t batch, kN, n, base_log, level;
 };
 
+// Tensor-core key switch: digit and limb tiles in the MMA layout.
+struct KsTcArgs {
+  const uint16_t *a_tiles;  // [m_tiles][k_steps][128 x 64] bf16 digits
+  const uint16_t *b_tiles;  // [n_tiles][k_steps][256 x 64] bf16 key limbs
+  const uint64_t *big;      // [batch][kN+1]
+  uint64_t *out;            // [batch][n+1]
+  uint32_t *err_flag;       // set to 2 when a wait gives up
+  uint32_t batch, kN, n, k_steps, limbs;
+};
+
 struct TraceArgs {
   const uint64_t *glwe_in;  // [batch][2][N]
   uint64_t *glwe_out;       // [batch][2][N]
@@ -80,6 +90,12 @@ cudaError_t launch_trace(const TraceArgs &a, uint32_t logN, cudaStream_t s);
 cudaError_t launch_plaintext_mul(const TraceArgs &a, uint32_t logN, cudaStream_t s);
 cudaError_t launch_monomial_acc(uint64_t *R, const uint64_t *r, uint32_t count, uint32_t logN, uint32_t e, bool first,
                                 cudaStream_t s);
+uint32_t ks_tc_limbs(uint32_t kN, uint32_t level, uint32_t base_log);  // 8, 16, or 0 (not exact)
+size_t ks_tc_b_words16(uint32_t kN, uint32_t level, uint32_t n, uint32_t limbs);
+size_t ks_tc_a_words16(uint32_t batch, uint32_t kN, uint32_t level);
+cudaError_t launch_ks_limbs(const uint64_t *ksk, uint16_t *b_tiles, uint32_t kN, uint32_t level, uint32_t n,
+                            uint32_t limbs, cudaStream_t s);
+cudaError_t launch_keyswitch_tc(const KsTcArgs &a, uint32_t base_log, uint32_t level, cudaStream_t s);
 cudaError_t launch_ksk_corr(const uint64_t *ksk, uint64_t *corr, uint32_t rows, uint32_t n, uint32_t base_log,
                             cudaStream_t s);
 

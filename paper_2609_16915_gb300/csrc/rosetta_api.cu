@@ -170,6 +170,34 @@ BrArgs br_args(const rosetta_ctx *c, const uint64_t *in, uint32_t batch, const u
   return a;
 }
 
+// Batches from this size on take the tensor-core key switch (when exact for
+// the parameters); smaller ones the split-K CUDA-core kernel.
+constexpr uint32_t kKsTcMinBatch = 256;
+
+KsArgs ks_args(const rosetta_ctx *c, const uint64_t *big, uint32_t batch, uint64_t *out);
+
+cudaError_t run_keyswitch(rosetta_ctx *c, const uint64_t *big, uint32_t batch, uint64_t *out, cudaStream_t s) {
+  const rosetta_params &p = c->prm;
+  const uint32_t kN = p.glwe_dim * p.poly_size;
+  if (c->ks_limbs && c->d_ks_b && batch >= kKsTcMinBatch) {
+    const size_t words16 = ks_tc_a_words16(batch, kN, p.ks_level);
+    if (ensure(&c->d_ks_a, &c->ks_a_cap, (words16 + 3) / 4, s) != ROSETTA_OK) return cudaErrorMemoryAllocation;
+    KsTcArgs a{};
+    a.a_tiles = reinterpret_cast<const uint16_t *>(c->d_ks_a);
+    a.b_tiles = c->d_ks_b;
+    a.big = big;
+    a.out = out;
+    a.err_flag = c->d_err;
+    a.batch = batch;
+    a.kN = kN;
+    a.n = p.lwe_dim;
+    a.k_steps = kN * p.ks_level / 64;
+    a.limbs = c->ks_limbs;
+    return launch_keyswitch_tc(a, p.ks_base_log, p.ks_level, s);
+  }
+  return launch_keyswitch(ks_args(c, big, batch, out), s);
+}
+
 KsArgs ks_args(const rosetta_ctx *c, const uint64_t *big, uint32_t batch, uint64_t *out) {
   KsArgs k{};
   k.big = big;
@@ -347,6 +375,14 @@ int rosetta_upload_ksk(rosetta_ctx *c, const uint64_t *ksk, size_t n_words, int 
   if (e != cudaSuccess) return cuda_fail(e);
   e = launch_ksk_corr(c->d_ksk, c->d_corr, (uint32_t)rows, p.lwe_dim, p.ks_base_log, s);
   if (e != cudaSuccess) return cuda_fail(e);
+  // limb tiles for the tensor-core key switch, where its fp32 sums are exact
+  const uint32_t kN = p.glwe_dim * p.poly_size;
+  c->ks_limbs = ks_tc_limbs(kN, p.ks_level, p.ks_base_log);
+  if (c->ks_limbs) {
+    if (!c->d_ks_b) e = cudaMalloc(&c->d_ks_b, ks_tc_b_words16(kN, p.ks_level, p.lwe_dim, c->ks_limbs) * 2);
+    if (e == cudaSuccess) e = launch_ks_limbs(c->d_ksk, c->d_ks_b, kN, p.ks_level, p.lwe_dim, c->ks_limbs, s);
+    if (e != cudaSuccess) return cuda_fail(e);
+  }
   if (!src_is_device) {
     e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) return cuda_fail(e);
@@ -382,7 +418,7 @@ int rosetta_keyswitch_batch(rosetta_ctx *c, const uint64_t *lwe_big_in, uint32_t
   Staged st;
   int r = stage_io(c, lwe_big_in, big_words(c), batch, nullptr, lwe_out, lwe_words(c), s, &st);
   if (r != ROSETTA_OK) return r;
-  cudaError_t e = launch_keyswitch(ks_args(c, st.in, batch, st.out), s);
+  cudaError_t e = run_keyswitch(c, st.in, batch, st.out, s);
   if (e != cudaSuccess) return cuda_fail(e);
   return finish_io(c, lwe_out, lwe_words(c), batch, st, s);
 }
@@ -402,7 +438,7 @@ int rosetta_pbs_batch(rosetta_ctx *c, const uint64_t *lwe_in, uint32_t batch, co
   if (r != ROSETTA_OK) return r;
   cudaError_t e = launch_blind_rotate(br_args(c, st.in, batch, st.lut, c->d_big), c->logN, c->dig16, s);
   if (e != cudaSuccess) return cuda_fail(e);
-  e = launch_keyswitch(ks_args(c, c->d_big, batch, st.out), s);
+  e = run_keyswitch(c, c->d_big, batch, st.out, s);
   if (e != cudaSuccess) return cuda_fail(e);
   return finish_io(c, lwe_out, lwe_words(c), batch, st, s);
 }
@@ -429,7 +465,7 @@ int rosetta_pbs_batch_multi_lut(rosetta_ctx *c, const uint64_t *lwe_in, uint32_t
   a.num_luts = num_luts;
   cudaError_t e = launch_blind_rotate(a, c->logN, c->dig16, s);
   if (e != cudaSuccess) return cuda_fail(e);
-  e = launch_keyswitch(ks_args(c, c->d_big, batch, st.out), s);
+  e = run_keyswitch(c, c->d_big, batch, st.out, s);
   if (e != cudaSuccess) return cuda_fail(e);
   return finish_io(c, lwe_out, lwe_words(c), batch, st, s);
 }
@@ -636,7 +672,7 @@ int rosetta_segmented_lookup_batch(rosetta_ctx *c, const uint64_t *glwe_x, const
     a.glwe_in = T;
     e = launch_blind_rotate(a, c->logN, c->dig16, s);
   }
-  if (e == cudaSuccess) e = launch_keyswitch(ks_args(c, c->d_big, batch, I), s);
+  if (e == cudaSuccess) e = run_keyswitch(c, c->d_big, batch, I, s);
   // Step 3, phase 1: r_s = a_s(X) [[x]] + b_s(X), rotated by [[I]], traced, and
   // accumulated as R = sum_s X^(s box) r_s
   const uint32_t seg_box = static_cast<uint32_t>(N / nseg);
@@ -674,7 +710,8 @@ int rosetta_sync_status(rosetta_ctx *c, void *stream) {
   e = cudaMemcpy(&flag, c->d_err, sizeof(flag), cudaMemcpyDeviceToHost);
   if (e == cudaSuccess && flag) e = cudaMemset(c->d_err, 0, sizeof(flag));
   if (e != cudaSuccess) return cuda_fail(e);
-  return flag ? ROSETTA_ERR_INVALID_ARG : ROSETTA_OK;
+  // 1: a LUT index out of range; 2: a bounded device-side wait gave up
+  return flag == 2 ? ROSETTA_ERR_TIMEOUT : (flag ? ROSETTA_ERR_INVALID_ARG : ROSETTA_OK);
 }
 
 void rosetta_destroy(rosetta_ctx *c) {
@@ -685,6 +722,8 @@ void rosetta_destroy(rosetta_ctx *c) {
   cudaFree(c->d_bsk);
   cudaFree(c->d_ksk);
   cudaFree(c->d_corr);
+  cudaFree(c->d_ks_b);
+  cudaFree(c->d_ks_a);
   cudaFree(c->d_big);
   cudaFree(c->d_in);
   cudaFree(c->d_out);

@@ -153,6 +153,19 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
   const uint64_t round_add = bits >= 64 ? 0 : (1ull << (63 - bits));
   const uint32_t round_sh = bits >= 64 ? 0 : 64 - bits;
 
+  // With one gadget level and N <= 2048 the remote bases of this thread's
+  // digit and residue slots in each CTA are kept across the steps (measured
+  // 1.5 % faster at N = 2048); elsewhere the registers are needed for the
+  // transforms.
+  constexpr bool HOIST = (LEV == 1 && LOGN <= 11);
+  uint32_t dig_r[4], res_r[4];
+  if constexpr (HOIST) {
+#pragma unroll
+    for (int r = 0; r < 4; ++r) {
+      dig_r[r] = dsmem_map(dig_s + tau * static_cast<uint32_t>(sizeof(DigT)), r);
+      res_r[r] = dsmem_map(res_s + (rank * 2 * Q + tau) * 4u, r);
+    }
+  }
   for (uint32_t i = 0; i < a.n; ++i) {
     const uint32_t at = atil[i];
     if (at == 0) continue;  // X^0 ACC - ACC = 0: the step adds nothing
@@ -201,7 +214,9 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
       for (int pp = 0; pp < 2; ++pp)
 #pragma unroll
         for (int q = 0; q < E; ++q) {
-          const uint32_t ad = dsmem_map(dig_s + ((r0 + pp) * Q + tau + (q % QE) * T) * sizeof(DigT), q / QE);
+          const uint32_t ad =
+              HOIST ? dig_r[q / QE] + ((r0 + pp) * Q + (q % QE) * T) * static_cast<uint32_t>(sizeof(DigT))
+                    : dsmem_map(dig_s + ((r0 + pp) * Q + tau + (q % QE) * T) * sizeof(DigT), q / QE);
           const int32_t d = DIG16 ? dsmem_ld_s16(ad) : dsmem_ld_s32(ad);
           x[pp][q] = static_cast<uint32_t>(d + static_cast<int32_t>(p));  // in (0, 2p)
         }
@@ -240,7 +255,9 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
 #pragma unroll
       for (int q = 0; q < E; ++q) {
         const uint32_t y = shoup_mul(oh[c][q], crt_c, crt_cs, p);  // [0, 2p)
-        dsmem_st_u32(dsmem_map(res_s + ((rank * 2 + c) * Q + tau + (q % QE) * T) * 4u, q / QE), y);
+        dsmem_st_u32(HOIST ? res_r[q / QE] + (c * Q + (q % QE) * T) * 4u
+                           : dsmem_map(res_s + ((rank * 2 + c) * Q + tau + (q % QE) * T) * 4u, q / QE),
+                     y);
       }
     cluster.sync();
 

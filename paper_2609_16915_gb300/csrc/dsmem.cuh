@@ -9,7 +9,8 @@ __device__ __forceinline__ uint32_t smem_addr(const void *p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
 
-// Address of the same shared-memory location in CTA `rank` of the cluster.
+// Address of the same shared-memory location in CTA `rank` of the cluster
+// (the windows are linear: mapa(a + off, r) = mapa(a, r) + off).
 __device__ __forceinline__ uint32_t dsmem_map(uint32_t local, uint32_t rank) {
   uint32_t r;
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(local), "r"(rank));

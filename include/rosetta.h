@@ -252,6 +252,15 @@ int rosetta_segmented_lookup_batch(rosetta_ctx *ctx, const uint64_t *glwe_x, con
 int rosetta_pbs_batch_noalloc(rosetta_ctx *ctx, const uint64_t *lwe_in, uint32_t batch,
                               const uint64_t *lut, uint64_t *lwe_out, void *stream);
 
+/* Self-test of the bounded device-side waits (no counterpart in the paper):
+ * launches one thread that waits on a barrier nothing completes, gives up
+ * after about limit_us microseconds (1 .. 10^6) and raises the context's
+ * error flag the way the tensor-core key switch does when one of its waits
+ * expires; rosetta_sync_status then returns TIMEOUT once and the context
+ * stays usable.  No fault, no hang: the wait is bounded.  Errors:
+ * INVALID_ARG, CUDA. */
+int rosetta_selftest_wait_timeout(rosetta_ctx *ctx, uint32_t limit_us, void *stream);
+
 /* Wait for all work on `stream` and report any deferred execution error
  * (CUDA; TIMEOUT when a bounded wait of the tensor-core key switch gave up;
  * INVALID_ARG for an out-of-range LUT index seen by

@@ -24,6 +24,7 @@ EXPORTS = ("rosetta_params_init", "rosetta_upload_bsk", "rosetta_upload_ksk", "r
            "rosetta_blind_rotate_extract_batch", "rosetta_keyswitch_batch", "rosetta_pbs_batch_multi_lut",
            "rosetta_blind_rotate_glwe_batch", "rosetta_upload_trace_keys", "rosetta_trace_batch",
            "rosetta_plaintext_mul_batch", "rosetta_upload_lookup_table", "rosetta_segmented_lookup_batch",
+           "rosetta_selftest_wait_timeout",
            "rosetta_pbs_batch_noalloc",
            "rosetta_sync_status", "rosetta_destroy", "rosetta_status_string")
 
@@ -66,6 +67,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     L.rosetta_plaintext_mul_batch.argtypes = [vp, u64p, u32, u64p, u64p, u64p, vp]
     L.rosetta_upload_lookup_table.argtypes = [vp, u32, u64p, u64p, u64p, u64p, vp]
     L.rosetta_segmented_lookup_batch.argtypes = [vp, u64p, u64p, u32, u64p, vp]
+    L.rosetta_selftest_wait_timeout.argtypes = [vp, u32, vp]
     L.rosetta_sync_status.argtypes = [vp, vp]
     L.rosetta_destroy.argtypes = [vp]
     L.rosetta_destroy.restype = None
@@ -227,6 +229,11 @@ class Context:
                                                      _ptr(glwe_out), _stream(stream)))
         return glwe_out
 
+    def rosetta_selftest_wait_timeout(self, limit_us=10000, stream=None):
+        """Make one bounded device wait expire (reported by sync_status as TIMEOUT)."""
+        _check("rosetta_selftest_wait_timeout",
+               load().rosetta_selftest_wait_timeout(self._h, limit_us, _stream(stream)))
+
     def rosetta_pbs_batch_noalloc(self, lwe_in, lut, lwe_out, stream=None):
         """rosetta_pbs_batch without any device allocation in the call (fixed
         in-library scratch; device buffers only, bounded batch)."""
@@ -251,4 +258,5 @@ class Context:
     plaintext_mul_batch = rosetta_plaintext_mul_batch
     upload_lookup_table = rosetta_upload_lookup_table
     segmented_lookup_batch = rosetta_segmented_lookup_batch
+    selftest_wait_timeout = rosetta_selftest_wait_timeout
     sync_status = rosetta_sync_status

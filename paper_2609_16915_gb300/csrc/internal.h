@@ -96,6 +96,7 @@ size_t ks_tc_a_words16(uint32_t batch, uint32_t kN, uint32_t level);
 cudaError_t launch_ks_limbs(const uint64_t *ksk, uint16_t *b_tiles, uint32_t kN, uint32_t level, uint32_t n,
                             uint32_t limbs, cudaStream_t s);
 cudaError_t launch_keyswitch_tc(const KsTcArgs &a, uint32_t base_log, uint32_t level, cudaStream_t s);
+cudaError_t launch_wait_selftest(uint32_t *err_flag, uint32_t limit_us, cudaStream_t s);
 cudaError_t launch_ksk_corr(const uint64_t *ksk, uint64_t *corr, uint32_t rows, uint32_t n, uint32_t base_log,
                             cudaStream_t s);
 

@@ -71,7 +71,7 @@ __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
 }
 
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, long long limit = kWaitCycles) {
   const long long t0 = clock64();
   while (true) {
     uint32_t done;
@@ -81,7 +81,7 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
         : "r"(bar), "r"(parity)
         : "memory");
     if (done) return true;
-    if (clock64() - t0 > kWaitCycles) return false;
+    if (clock64() - t0 > limit) return false;
   }
 }
 
@@ -295,6 +295,22 @@ __global__ void __launch_bounds__(TC_THREADS, 1) ks_tc_kernel(const KsTcArgs a) 
   __syncthreads();
   if (warp == 0)
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TMEM_COLS) : "memory");
+}
+
+// Self-test of the bounded-wait path: one thread waits on an mbarrier that
+// nothing completes, gives up after `limit` cycles and reports it through the
+// error flag exactly as ks_tc_kernel does.
+__global__ void wait_selftest_kernel(uint32_t *err_flag, long long limit) {
+  __shared__ __align__(8) uint64_t bar;
+  const uint32_t b = smem_addr(&bar);
+  mbar_init(b, 1);
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  if (!mbar_wait(b, 0, limit)) atomicExch(err_flag, 2u);
+}
+
+cudaError_t launch_wait_selftest(uint32_t *err_flag, uint32_t limit_us, cudaStream_t s) {
+  wait_selftest_kernel<<<1, 1, 0, s>>>(err_flag, static_cast<long long>(limit_us) * 2000);  // ~2 GHz
+  return cudaGetLastError();
 }
 
 // ---------------------------------------------------------------------------- host side

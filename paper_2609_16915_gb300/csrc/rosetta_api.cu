@@ -699,6 +699,13 @@ int rosetta_segmented_lookup_batch(rosetta_ctx *c, const uint64_t *glwe_x, const
   return e == cudaSuccess ? ROSETTA_OK : cuda_fail(e);
 }
 
+int rosetta_selftest_wait_timeout(rosetta_ctx *c, uint32_t limit_us, void *stream) {
+  if (!c || limit_us == 0 || limit_us > 1000000) return ROSETTA_ERR_INVALID_ARG;
+  if (cudaSetDevice(c->device) != cudaSuccess) return ROSETTA_ERR_CUDA;
+  cudaError_t e = launch_wait_selftest(c->d_err, limit_us, as_stream(stream));
+  return e == cudaSuccess ? ROSETTA_OK : cuda_fail(e);
+}
+
 int rosetta_sync_status(rosetta_ctx *c, void *stream) {
   if (!c) return ROSETTA_ERR_INVALID_ARG;
   if (cudaSetDevice(c->device) != cudaSuccess) return ROSETTA_ERR_CUDA;

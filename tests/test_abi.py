@@ -71,3 +71,27 @@ def test_argument_checks_before_cuda(lib):
     assert lib.rosetta_keyswitch_batch(None, None, 0, None, None) == -1
     assert lib.rosetta_sync_status(None, None) == -1
     lib.rosetta_destroy(None)
+
+
+def build_c_client(out_path):
+    """Compile tests/c_abi_demo.c, a plain C99 program that uses the library
+    through include/rosetta.h alone, and link it against librosetta.so."""
+    import shutil
+    import subprocess
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("gcc not installed")
+    here = os.path.dirname(os.path.abspath(__file__))
+    root = os.path.dirname(here)
+    pkg = os.path.join(root, "paper_2609_16915_gb300")
+    cmd = [gcc, "-std=c99", "-Wall", "-Wextra", "-Werror", "-I", os.path.join(root, "include"),
+           os.path.join(here, "c_abi_demo.c"), "-L", pkg, "-lrosetta", f"-Wl,-rpath,{pkg}",
+           "-L/usr/local/cuda/lib64", "-o", out_path]
+    r = subprocess.run(cmd, capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
+    return out_path
+
+
+def test_c_client_compiles_and_links(lib, tmp_path):
+    """The header is plain C and the library links from C without CUDA headers."""
+    assert os.path.exists(build_c_client(str(tmp_path / "c_abi_demo")))

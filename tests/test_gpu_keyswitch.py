@@ -50,3 +50,21 @@ def test_keyswitch_extreme_digits():
     ctx = R.Context(p)
     ctx.upload_ksk(G.to_dev(ksk))
     assert np.array_equal(G.gpu_keyswitch(ctx, p, big), O.keyswitch_batch(p, ksk, big))
+
+
+def test_expired_wait_is_reported_and_the_context_stays_usable():
+    """A bounded wait that nothing completes gives up, sync_status reports
+    TIMEOUT once, and the next key switch on the same context is exact."""
+    import paper_2609_16915_gb300 as R
+    p = W.CONFIGS["standard"]
+    _, ksk = W.uniform_keys(p, seed=93)
+    ctx = R.Context(p)
+    ctx.upload_ksk(G.to_dev(ksk))
+    ctx.sync_status()
+    ctx.selftest_wait_timeout(20000)
+    with pytest.raises(R.RosettaError) as e:
+        ctx.sync_status()
+    assert e.value.status == -6
+    ctx.sync_status()                                # reported once, then cleared
+    big = W.uniform_u64((300, p.kN + 1), W.rng(p.seed, "sample", 97))
+    assert np.array_equal(G.gpu_keyswitch(ctx, p, big), O.keyswitch_batch(p, ksk, big))

@@ -290,3 +290,26 @@ def test_error_codes():
     st = L.rosetta_upload_bsk(ctx._h, G.to_dev(keys.bsk).data_ptr(), keys.bsk.size - 1, 1, None)
     assert st == -1                               # wrong key size
     ctx.sync_status()
+
+
+def test_c_client_bootstraps_like_the_oracle(tmp_path):
+    """A C99 program (tests/c_abi_demo.c) drives the library with host buffers:
+    same words as the oracle."""
+    import subprocess
+    from tests.test_abi import build_c_client
+    p = W.CONFIGS["tiny"]
+    keys = real_keys("tiny")
+    lwe = keys.encrypt(W.cipher_draws(p, 21, sub=31))
+    lut = W.lut_torus(p)
+    inp, outp = tmp_path / "in.bin", tmp_path / "out.bin"
+    head = np.array([p.n, p.k, p.N, p.pbs_base_log, p.pbs_level, p.ks_base_log, p.ks_level, p.msg_bits, 0,
+                     lwe.shape[0]], np.uint32)
+    with open(inp, "wb") as f:
+        for a in (head, keys.bsk, keys.ksk, lut, lwe):
+            f.write(np.ascontiguousarray(a).tobytes())
+    exe = build_c_client(str(tmp_path / "c_abi_demo"))
+    r = subprocess.run([exe, str(inp), str(outp)], capture_output=True, text=True, timeout=300)
+    assert r.returncode == 0, r.stderr
+    got = np.fromfile(outp, dtype=np.uint64).reshape(lwe.shape)
+    assert np.array_equal(got, O.pbs_batch(p, keys.bsk, keys.ksk, lwe, lut))
+    assert np.array_equal(keys.decrypt(got), W.lut_codes(p)[W.cipher_draws(p, 21, sub=31).codes])

@@ -49,7 +49,11 @@
  * Execution errors surface at rosetta_sync_status or at the next call.
  * No function falls back to the CPU.
  *
- * Threading.  A context may be used from one host thread at a time.
+ * Threading.  A context may be used from one host thread at a time.  Its
+ * scratch buffers (extracted ciphertexts, staging, key-switch digit tiles,
+ * lookup intermediates) are shared by its calls, which are ordered only on
+ * one stream: work issued through one context on two streams at once must be
+ * synchronised by the caller (or use one context per stream).
  */
 #ifndef ROSETTA_H
 #define ROSETTA_H

@@ -329,3 +329,29 @@ def test_lookup_argument_checks():
     with pytest.raises(R.RosettaError) as e:        # tables in device memory
         ctx.upload_lookup_table(G.to_dev(zu), zu, np.zeros((2, p.N), np.int64), np.zeros((2, p.N), np.uint64))
     assert e.value.status == -1
+
+
+def test_lookup_one_interval_per_coefficient_on_gpu():
+    """N_br = N (boxes of one coefficient, the paper's setting): GPU words =
+    oracle words, decrypting to the cleartext lookup."""
+    from paper_2609_16915_gb300 import segmented as SG
+    from tests import lookup_util as LU
+    p = W.CONFIGS["lookup_small"]
+    keys = O.Keys(p, W.key_draws(p))
+    tk = LU.trace_keys(p, keys.glwe_key)
+    lut = SG.build(SG.FUNCTIONS["reciprocal"], [0.1, 0.5, 2.0], p.N)
+    enc = SG.encode(lut, p.N, LU.DX, LU.DR)
+    xs = LU.sample_points(lut, 8, 19)
+    segs = [SG.segment_index(lut, x) for x in xs]
+    glwe, lwe = LU.encrypt_inputs(p, keys, xs, segs, lut.n_seg, sub=4)
+    tables = (enc.p_hat, enc.q_hat, enc.a_hat, enc.b_hat)
+    ctx = _lookup_ctx(p, keys.bsk, keys.ksk, tk, LU.TRACE_BASE_LOG, LU.TRACE_LEVEL, tables)
+    out = G.empty_dev(len(xs), 2, p.N)
+    ctx.segmented_lookup_batch(G.to_dev(glwe), G.to_dev(lwe), out)
+    ctx.sync_status()
+    got = G.to_host(out)
+    assert np.array_equal(got, O.segmented_lookup_batch(p, keys.bsk, keys.ksk, tk, LU.TRACE_BASE_LOG,
+                                                        LU.TRACE_LEVEL, glwe, lwe, *tables))
+    S = keys.glwe_key.reshape(1, -1)
+    for b, x in enumerate(xs):
+        assert SG.decode(O.glwe_phase(S, got[b])[0], enc) == pytest.approx(SG.lookup(lut, x), abs=1e-2)

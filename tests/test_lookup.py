@@ -142,3 +142,23 @@ def test_composed_lookup_decrypts_to_the_paper_value(small_setup):
     assert got[0] == pytest.approx(G["value"], abs=2e-3)
     for x, v in zip(xs, got):
         assert v == pytest.approx(SG.lookup(lut, x), abs=1e-2), x
+
+
+def test_composed_lookup_one_interval_per_coefficient(small_setup):
+    """N_br = N (the paper's setting: every ring coefficient is an interval,
+    boxes of one coefficient): the encrypted lookup still decrypts to the
+    cleartext lookup, now with N intervals per segment."""
+    p, keys, tk, _, _ = small_setup
+    lut = SG.build(SG.FUNCTIONS["reciprocal"], [0.1, 0.5, 2.0], p.N)
+    enc = SG.encode(lut, p.N, LU.DX, LU.DR)
+    xs = LU.sample_points(lut, 6, 17)
+    segs = [SG.segment_index(lut, x) for x in xs]
+    glwe, lwe = LU.encrypt_inputs(p, keys, xs, segs, lut.n_seg, sub=3)
+    out = O.segmented_lookup_batch(p, keys.bsk, keys.ksk, tk, LU.TRACE_BASE_LOG, LU.TRACE_LEVEL, glwe, lwe,
+                                   enc.p_hat, enc.q_hat, enc.a_hat, enc.b_hat)
+    S = keys.glwe_key.reshape(1, -1)
+    for b, x in enumerate(xs):
+        v = SG.decode(O.glwe_phase(S, out[b])[0], enc)
+        assert v == pytest.approx(SG.lookup(lut, x), abs=1e-2), x
+        # 512 intervals per segment: within the slope quantisation (2^-9 |x|) of 1/x
+        assert v == pytest.approx(1.0 / x, abs=1e-2), x

@@ -92,7 +92,10 @@ typedef struct {
 /* Create a context on CUDA device `cuda_device` for parameter set *p.
  * Computes the NTT primes' twiddle tables and CRT constants and allocates
  * scratch for p->max_batch ciphertexts.  *out receives the context (NULL on
- * error).  Errors: INVALID_ARG (NULL), UNSUPPORTED_PARAMS, CUDA, OOM. */
+ * error).  UNSUPPORTED_PARAMS also when the exact external product would
+ * not fit the four NTT primes: log2((k+1) l N 2^(beta-1) 2^63) + 1 must not
+ * exceed 111 (their product is about 2^111.99).  Errors: INVALID_ARG (NULL),
+ * UNSUPPORTED_PARAMS, CUDA, OOM. */
 int rosetta_params_init(rosetta_ctx **out, const rosetta_params *p, int cuda_device);
 
 /* Upload the raw bootstrapping key (layout above, n_words =

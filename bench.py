@@ -12,7 +12,8 @@ the host cores instead (the reference arm: a deliberately plain program).
 `--path lookup` measures the encrypted segmented lookup instead (the
 lookup protocol's Steps 2 and 3 composed from plaintext products, blind
 rotations of GLWE test polynomials, a key switch and RLWE traces) on the
-same ring, four segments, one line of its own.
+same ring, four segments, one line of its own; `--path multi_lut` the PBS
+with a LUT per ciphertext (four LUTs in one launch).
 """
 
 from __future__ import annotations
@@ -332,6 +333,62 @@ def run_lookup(args, p, batch, torch, dev, R, clock_sampler):
     print(json.dumps(line), flush=True)
 
 
+# ---------------------------------------------------------------------------- many-LUT path
+
+MULTI_METRIC = "PBS/sec with a LUT per ciphertext (4 LUTs in one launch) on 1 GB300"
+
+
+def run_multi_lut(args, p, batch, torch, dev, R, clock_sampler):
+    """Throughput of rosetta_pbs_batch_multi_lut: four LUTs (the workload's
+    and three shifted copies) assigned round-robin to the ciphertexts."""
+    def d(a):
+        return torch.from_numpy(np.ascontiguousarray(a).view(np.int64)).to(dev)
+
+    bsk, ksk = W.uniform_keys(p)
+    ctx = R.Context(p, device=dev.index or 0, max_batch=batch)
+    ctx.upload_bsk(d(bsk))
+    ctx.upload_ksk(d(ksk))
+    del bsk, ksk
+    codes = W.lut_codes(p)
+    luts = d(np.stack([W.lut_torus(p, np.roll(codes, r)) for r in range(4)]))
+    idx = torch.from_numpy((np.arange(batch) % 4).astype(np.int32)).to(dev)
+    lwe = d(W.uniform_ciphertexts(p, batch, sub=9))
+    out = torch.empty((batch, p.n + 1), dtype=torch.int64, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.int32, device=dev)
+    for _ in range(max(3, args.warmup)):
+        ctx.pbs_batch_multi_lut(lwe, luts, idx, out, stream)
+    ctx.sync_status(stream)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    torch.cuda.synchronize(dev)
+    with clock_sampler(dev.index or 0) as clk:
+        for s_ in range(args.steps):
+            flush.zero_()
+            ev[s_][0].record(stream)
+            ctx.pbs_batch_multi_lut(lwe, luts, idx, out, stream)
+            ev[s_][1].record(stream)
+        torch.cuda.synchronize(dev)
+    ctx.sync_status(stream)
+    total_ms = sum(a.elapsed_time(b) for a, b in ev)
+    value = batch * args.steps / (total_ms / 1e3)
+    br_ops, ks_ops = int_ops_per_pbs(p)
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    alu_peak = sms * 128 * peaks().get("sm_max_mhz", 2070.0) * 1e6 / 1e12
+    achieved = br_ops * batch * args.steps / (total_ms / 1e3) / 1e12
+    line = {
+        "metric": MULTI_METRIC, "value": value, "unit": "PBS/s", "n_gpus": 1, "steps": args.steps,
+        "warmup": max(3, args.warmup), "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "u64", "data": "synthetic",
+        "config": {"workload": describe(p, batch) + ", 4 LUTs round-robin", "batch": batch,
+                   "l2": "flushed between steps (256 MB write)", "keys": "uniform words, resident"},
+        "roofline": {"bound": "alu", "kernel": "blind_rotate_kernel + key switch (whole step)", "achieved": achieved,
+                     "peak": alu_peak, "unit": "Tops/s (int32)", "frac": achieved / alu_peak, "traffic": None},
+        "gpu_launches": (3 if ks_tensor_limbs(p, batch) else 2) * args.steps,
+        "clocks": clk.summary(),
+    }
+    print(json.dumps(line), flush=True)
+
+
 # ---------------------------------------------------------------------------- GPU arm
 
 def main():
@@ -344,19 +401,21 @@ def main():
     ap.add_argument("--batch", type=int, default=0, help="override the workload's batch")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-sample", type=int, default=0, help="oracle sample size (default: host cores)")
-    ap.add_argument("--path", default="pbs", choices=["pbs", "lookup"])
+    ap.add_argument("--path", default="pbs", choices=["pbs", "lookup", "multi_lut"])
     args = ap.parse_args()
     p = W.CONFIGS[args.config]
     batch = args.batch or p.batch
     if args.impl == "reference":
         return run_reference(args, p, batch)
-    if args.path == "lookup":
+    if args.path in ("lookup", "multi_lut"):
         import torch
         import paper_2609_16915_gb300 as R
         R.load()
         dev = torch.device("cuda", 0)
         torch.cuda.set_device(dev)
-        return run_lookup(args, p, args.batch or 1024, torch, dev, R, ClockSampler)
+        if args.path == "lookup":
+            return run_lookup(args, p, args.batch or 1024, torch, dev, R, ClockSampler)
+        return run_multi_lut(args, p, batch, torch, dev, R, ClockSampler)
 
     import torch
     world = int(os.environ.get("WORLD_SIZE", "1"))

@@ -19,7 +19,7 @@
 // needs no exchange.
 //
 // Lazy ranges: forward input < 2p, output < 16p; inverse input < 4p, output
-// < 4p.  See the butterflies for the per-stage invariants.
+// < 8p.  See the butterflies for the per-stage invariants.
 #pragma once
 #include <stdint.h>
 
@@ -85,26 +85,30 @@ __device__ __forceinline__ void ct_bfly(uint32_t &X, uint32_t &Y, uint2 w, uint3
 __host__ __device__ constexpr bool fwd_stage_corrects(int s) { return s >= 7 && ((s - 7) % 4 == 0); }
 
 // Inverse (Gentleman-Sande) butterfly with inverse twiddle -w:
-// X' = X + Y, Y' = (X - Y)(-w) = (Y - X + 4p) w.  Inputs < 4p give X' < 8p,
-// brought below 4p when corr, and Y' < 2p.  Both inputs of an inverse
-// butterfly are outputs of the same kind (X' or Y') of the previous stage;
-// when they are Y' outputs (< 2p) their sum is already below 4p and the
-// correction is skipped.
-__device__ __forceinline__ void gs_bfly(uint32_t &X, uint32_t &Y, uint2 w, uint32_t p, uint32_t four_p, bool corr) {
+// X' = X + Y, Y' = (X - Y)(-w) = (Y - X + 8p) w.  Inputs < 8p give
+// X' < 16p, brought below 8p when corr, and Y' < 2p (16p < 2^32).
+__device__ __forceinline__ void gs_bfly(uint32_t &X, uint32_t &Y, uint2 w, uint32_t p, uint32_t eight_p, bool corr) {
   const uint32_t s = X + Y;
-  const uint32_t d = Y - X + four_p;
-  X = corr ? cond_sub(s, four_p) : s;  // corr is a constant after unrolling
+  const uint32_t d = Y - X + eight_p;
+  X = corr ? cond_sub(s, eight_p) : s;  // corr is a constant after unrolling
   Y = shoup_mul(d, w.x, w.y, p);
 }
 
 // Does inverse stage S (inside the pass (S0, H), U = S - S0) need the
-// correction for the butterfly at register position q?  Its inputs come from
-// stage S+1, where the element at q was an X' output iff bit (H - U - 2) of q
-// is 0.  The first stage of every pass (U = H - 1) looks at a bit outside q
-// and always corrects.
-template <int H, int U>
+// correction for the butterfly at register position q?  Both inputs of an
+// inverse butterfly are outputs of the same kind (X' or Y') of stage S+1:
+// X' outputs iff bit (H - U - 2) of q is 0.  Y' inputs (< 2p) give X' < 4p:
+// no correction.  X' inputs are below 8p, or below 4p when their own
+// butterfly at stage S+2 had Y' inputs (bit (H - U - 3) of q is 1, known
+// when S+2 lies in the same pass): then X' < 8p needs no correction either.
+// The first stage of a pass sees inputs of unknown kind and corrects, except
+// the very first inverse stage (LAST pass), whose inputs are all below 4p.
+template <bool LAST, int H, int U>
 __host__ __device__ constexpr bool inv_corrects(int q) {
-  return U >= H - 1 ? true : ((q >> (H - U - 2)) & 1) == 0;
+  if (U >= H - 1) return !LAST;
+  if (((q >> (H - U - 2)) & 1) != 0) return false;
+  if (U + 2 <= H - 1 && ((q >> (H - U - 3)) & 1) == 1) return false;
+  return true;
 }
 
 // Load CNT (a power of two) consecutive twiddle pairs starting at an index
@@ -166,7 +170,8 @@ __device__ __forceinline__ void fwd_stage(uint32_t (&x)[NP][E], const uint2 *__r
 
 template <int LOGN, int E, int NP, int S0, int H, int U>
 __device__ __forceinline__ void inv_stage(uint32_t (&x)[NP][E], const uint2 *__restrict__ tw, uint32_t tau,
-                                          uint32_t p, uint32_t four_p) {
+                                          uint32_t p, uint32_t eight_p) {
+  constexpr bool LAST = (S0 + H == LOGN);  // the pass the inverse starts with
   constexpr uint32_t N = 1u << LOGN;
   constexpr uint32_t SIG = N >> (S0 + H);
   constexpr int NB = E >> H;
@@ -186,7 +191,8 @@ __device__ __forceinline__ void inv_stage(uint32_t (&x)[NP][E], const uint2 *__r
         const int idx = CNT - 1 - ((b << U) + (q >> (H - U)));
 #pragma unroll
         for (int k = 0; k < NP; ++k)
-          gs_bfly(x[k][b * (1 << H) + q], x[k][b * (1 << H) + q + HALF], w[idx], p, four_p, inv_corrects<H, U>(q));
+          gs_bfly(x[k][b * (1 << H) + q], x[k][b * (1 << H) + q + HALF], w[idx], p, eight_p,
+                  inv_corrects<LAST, H, U>(q));
       }
   } else {
 #pragma unroll
@@ -199,7 +205,7 @@ __device__ __forceinline__ void inv_stage(uint32_t (&x)[NP][E], const uint2 *__r
         const uint2 w = tw[(2u << S) - 1u - G];
 #pragma unroll
         for (int k = 0; k < NP; ++k)
-          gs_bfly(x[k][b * (1 << H) + q], x[k][b * (1 << H) + q + HALF], w, p, four_p, inv_corrects<H, U>(q));
+          gs_bfly(x[k][b * (1 << H) + q], x[k][b * (1 << H) + q + HALF], w, p, eight_p, inv_corrects<LAST, H, U>(q));
       }
     }
   }
@@ -214,9 +220,9 @@ __device__ __forceinline__ void fwd_pass(uint32_t (&x)[NP][E], const uint2 *tw, 
 
 template <int LOGN, int E, int NP, int S0, int H, int U = H - 1>
 __device__ __forceinline__ void inv_pass(uint32_t (&x)[NP][E], const uint2 *tw, uint32_t tau, uint32_t p,
-                                         uint32_t four_p) {
-  inv_stage<LOGN, E, NP, S0, H, U>(x, tw, tau, p, four_p);
-  if constexpr (U > 0) inv_pass<LOGN, E, NP, S0, H, U - 1>(x, tw, tau, p, four_p);
+                                         uint32_t eight_p) {
+  inv_stage<LOGN, E, NP, S0, H, U>(x, tw, tau, p, eight_p);
+  if constexpr (U > 0) inv_pass<LOGN, E, NP, S0, H, U - 1>(x, tw, tau, p, eight_p);
 }
 
 // A pass whose butterfly groups span S elements keeps the data of every run of
@@ -349,7 +355,7 @@ __device__ __forceinline__ void ntt_inverse(uint32_t (&x)[NP][E], const uint2 *t
   using S = NttShape<LOGN, E>;
   constexpr int S0 = S::RAD * PASS;
   constexpr int H = S::template h<PASS>();
-  inv_pass<LOGN, E, NP, S0, H>(x, tw, tau, p, 4 * p);
+  inv_pass<LOGN, E, NP, S0, H>(x, tw, tau, p, 8 * p);
   if constexpr (PASS > 0) {
     exchange<LOGN, E, NP, XBUF, S0, H, S0 - S::RAD, S::RAD>(x, xb, tau);
     ntt_inverse<LOGN, E, NP, XBUF, PASS - 1>(x, tw, xb, tau, p);

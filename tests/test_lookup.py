@@ -162,3 +162,20 @@ def test_composed_lookup_one_interval_per_coefficient(small_setup):
         assert v == pytest.approx(SG.lookup(lut, x), abs=1e-2), x
         # 512 intervals per segment: within the slope quantisation (2^-9 |x|) of 1/x
         assert v == pytest.approx(1.0 / x, abs=1e-2), x
+
+
+@pytest.mark.parametrize("n_seg", [1, 2, 4, 8])
+def test_oracle_segment_boxes_select_their_segment(n_seg):
+    """Rotating the oracle's box polynomial of segment s left by s box + d
+    (|d| within half a box, the noise a blind rotation by [[S]] can add)
+    leaves 1 in the constant coefficient; its shift by another segment leaves 0."""
+    N = 64
+    box, h = N // n_seg, N // n_seg // 2
+    for s in range(n_seg):
+        b = np.array([x % Q for x in O.segment_box(s, n_seg, N).tolist()], np.uint64)
+        for d in range(-h, box - h):
+            rot = O.poly_monomial(b, (2 * N - (s * box + d)) % (2 * N))
+            assert int(rot[0]) == 1, (s, d)
+        for s2 in range(n_seg):
+            if s2 != s:
+                assert int(O.poly_monomial(b, (2 * N - s2 * box) % (2 * N))[0]) == 0

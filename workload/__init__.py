@@ -96,6 +96,12 @@ CONFIGS = {
                         glwe_sigma_log2=13, lut=("exp", -8.0, 0.0),
                         msg=("normal", 2.0, -8.0, 0.0), batch=1024, seed=5,
                         batches=(1, 64, 1024, 16384, 65536)),
+    # The paper's TFHE dimensions (n = 1024, N_br = 2048; Experimental Setup)
+    # on the 2^64 torus: PBS 2^23 x 1, KS 2^3 x 5, 4-bit GELU, batch 4096.
+    "paper_dims": Params("paper_dims", n=1024, k=1, N=2048, pbs_base_log=23, pbs_level=1,
+                         ks_base_log=3, ks_level=5, msg_bits=4, lwe_sigma_log2=47,
+                         glwe_sigma_log2=13, lut=("gelu", -4.0, 4.0), msg=("uniform",),
+                         batch=4096, seed=7),
     # Encrypted segmented lookup on a small ring (two traces multiply the
     # result by N^2, so the noise of a blind rotation must stay well below
     # 2^63 / N^2): n=64, N=512, PBS 2^8 x 6, KS 2^4 x 8, 1/x on [0.1, 2.0]

@@ -82,9 +82,9 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
   extern __shared__ __align__(16) unsigned char smem[];
   uint2 *tw = reinterpret_cast<uint2 *>(smem);                   // [N]
   uint64_t *acc = reinterpret_cast<uint64_t *>(tw + N);          // [2][Q]
-  uint32_t *res = reinterpret_cast<uint32_t *>(acc + 2 * Q);     // [4 primes][2][Q]
+  uint32_t *res = reinterpret_cast<uint32_t *>(acc + 2 * Q);     // [4 primes][T][2 comp][QE halves]
   uint32_t *xb = res + kPrimes * 2 * Q;                          // [XBUF][XB_WORDS]
-  DigT *dig = reinterpret_cast<DigT *>(xb + B::XBUF * S::XB_WORDS);  // [2l][Q]
+  DigT *dig = reinterpret_cast<DigT *>(xb + B::XBUF * S::XB_WORDS);  // [l row pairs][T][2][QE]
   const uint32_t level = LEV > 0 ? static_cast<uint32_t>(LEV) : a.level;
   uint16_t *atil = reinterpret_cast<uint16_t *>(dig + 2 * level * Q);  // [n+1]
 
@@ -153,8 +153,18 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
   const uint64_t round_add = bits >= 64 ? 0 : (1ull << (63 - bits));
   const uint32_t round_sh = bits >= 64 ? 0 : 64 - bits;
 
+  // Packed exchange layouts.  Owner thread tau holds the items (c, jl) =
+  // (m / QE, tau + (m % QE) T), m < ITEMS = 2 QE, and prime thread tau needs
+  // from owner o exactly the coefficients tau + h T (h < QE) of both
+  // components: so digits are stored as [row pair][tau][row parity][h] and
+  // residues as [prime][tau][component][h], and every transfer between a
+  // pair of threads is one 2 QE-word vector access.
+  static_assert(ITEMS == 2 * QE, "one packed group of 2 QE items per thread");
+  constexpr uint32_t GRP = 2 * QE;  // words per packed group
+  const uint32_t dig_t = dig_s + tau * GRP * static_cast<uint32_t>(sizeof(DigT));
+  const uint32_t res_t = res_s + (rank * T + tau) * GRP * 4u;
   // With one gadget level and N <= 2048 the remote bases of this thread's
-  // digit and residue slots in each CTA are kept across the steps (measured
+  // digit and residue groups in each CTA are kept across the steps (measured
   // 1.5 % faster at N = 2048); elsewhere the registers are needed for the
   // transforms.
   constexpr bool HOIST = (LEV == 1 && LOGN <= 11);
@@ -162,8 +172,8 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
   if constexpr (HOIST) {
 #pragma unroll
     for (int r = 0; r < 4; ++r) {
-      dig_r[r] = dsmem_map(dig_s + tau * static_cast<uint32_t>(sizeof(DigT)), r);
-      res_r[r] = dsmem_map(res_s + (rank * 2 * Q + tau) * 4u, r);
+      dig_r[r] = dsmem_map(dig_t, r);
+      res_r[r] = dsmem_map(res_t, r);
     }
   }
   for (uint32_t i = 0; i < a.n; ++i) {
@@ -181,6 +191,10 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
       const uint32_t e = (j + TWO_N - at) & (N - 1);
       v[m] = dsmem_ld_u64(dsmem_map(acc_s + (c * Q + (e % Q)) * 8u, e / Q));
     }
+    // with a compile-time level the packed groups are assembled in registers
+    // and written with one vector store each
+    constexpr int NGRP = LEV > 0 ? LEV : 1;
+    int32_t grp[NGRP][GRP];
 #pragma unroll
     for (int m = 0; m < ITEMS; ++m) {
       const uint32_t item = tau + m * T;
@@ -197,7 +211,25 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
           ds -= static_cast<int32_t>(Bmask + 1);
           cv += 1;
         }
-        dig[(c * level + l) * Q + jl] = static_cast<DigT>(ds);
+        const uint32_t r = c * level + l;  // row; h = m % QE
+        if constexpr (LEV > 0)
+          grp[r >> 1][(r & 1) * QE + (m % QE)] = ds;
+        else
+          dig[(((r >> 1) * T + tau) * 2 + (r & 1)) * QE + (m % QE)] = static_cast<DigT>(ds);
+      }
+    }
+    if constexpr (LEV > 0) {
+      static_assert(GRP == 4, "four digits per group");
+#pragma unroll
+      for (int P = 0; P < NGRP; ++P) {
+        DigT *g = dig + (P * T + tau) * GRP;
+        if constexpr (DIG16)
+          *reinterpret_cast<uint2 *>(g) =
+              make_uint2((static_cast<uint32_t>(grp[P][0]) & 0xFFFFu) | (static_cast<uint32_t>(grp[P][1]) << 16),
+                         (static_cast<uint32_t>(grp[P][2]) & 0xFFFFu) | (static_cast<uint32_t>(grp[P][3]) << 16));
+        else
+          *reinterpret_cast<uint4 *>(g) = make_uint4(static_cast<uint32_t>(grp[P][0]), static_cast<uint32_t>(grp[P][1]),
+                                                     static_cast<uint32_t>(grp[P][2]), static_cast<uint32_t>(grp[P][3]));
       }
     }
     cluster.sync();
@@ -208,18 +240,35 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
 #pragma unroll 1
     for (uint32_t r0 = 0; r0 < L2; r0 += 2) {
       // first-pass slot q of thread tau is coefficient tau + q N/E, owned by
-      // CTA q / QE at local index tau + (q % QE) T
+      // CTA o = q / QE at local index tau + (q % QE) T: one packed group of
+      // the row pair per owner
       uint32_t x[2][E];
+      const uint32_t pair_off = (r0 >> 1) * T * GRP * static_cast<uint32_t>(sizeof(DigT));
 #pragma unroll
-      for (int pp = 0; pp < 2; ++pp)
-#pragma unroll
-        for (int q = 0; q < E; ++q) {
-          const uint32_t ad =
-              HOIST ? dig_r[q / QE] + ((r0 + pp) * Q + (q % QE) * T) * static_cast<uint32_t>(sizeof(DigT))
-                    : dsmem_map(dig_s + ((r0 + pp) * Q + tau + (q % QE) * T) * sizeof(DigT), q / QE);
-          const int32_t d = DIG16 ? dsmem_ld_s16(ad) : dsmem_ld_s32(ad);
-          x[pp][q] = static_cast<uint32_t>(d + static_cast<int32_t>(p));  // in (0, 2p)
+      for (int o = 0; o < 4; ++o) {
+        const uint32_t ad = (HOIST ? dig_r[o] : dsmem_map(dig_t, o)) + pair_off;
+        int32_t d[GRP];
+        if constexpr (DIG16) {
+          static_assert(GRP == 4, "four 16-bit digits per group");
+          const uint2 w = dsmem_ld_v2_u32(ad);
+          d[0] = static_cast<int16_t>(w.x & 0xFFFFu);
+          d[1] = static_cast<int16_t>(w.x >> 16);
+          d[2] = static_cast<int16_t>(w.y & 0xFFFFu);
+          d[3] = static_cast<int16_t>(w.y >> 16);
+        } else {
+          static_assert(GRP == 4, "four 32-bit digits per group");
+          const uint4 w = dsmem_ld_v4_u32(ad);
+          d[0] = static_cast<int32_t>(w.x);
+          d[1] = static_cast<int32_t>(w.y);
+          d[2] = static_cast<int32_t>(w.z);
+          d[3] = static_cast<int32_t>(w.w);
         }
+#pragma unroll
+        for (int pp = 0; pp < 2; ++pp)
+#pragma unroll
+          for (int h = 0; h < QE; ++h)
+            x[pp][o * QE + h] = static_cast<uint32_t>(d[pp * QE + h] + static_cast<int32_t>(p));  // in (0, 2p)
+      }
       ntt_forward<LOGN, E, 2, B::XBUF>(x, tw, xb, tau, p);
       // BSK_i words of this prime for rows r0, r0+1, E per thread and
       // component, contiguous across the CTA (16-byte loads)
@@ -250,18 +299,30 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
       }
     }
     ntt_inverse<LOGN, E, 2, B::XBUF>(oh, tw, xb, tau, p);
+    // CRT-scaled residues, one packed group (component, h) per owner
 #pragma unroll
-    for (int c = 0; c < 2; ++c)
+    for (int o = 0; o < 4; ++o) {
+      static_assert(GRP == 4, "four residues per group");
+      uint32_t y[4];
 #pragma unroll
-      for (int q = 0; q < E; ++q) {
-        const uint32_t y = shoup_mul(oh[c][q], crt_c, crt_cs, p);  // [0, 2p)
-        dsmem_st_u32(HOIST ? res_r[q / QE] + (c * Q + (q % QE) * T) * 4u
-                           : dsmem_map(res_s + ((rank * 2 + c) * Q + tau + (q % QE) * T) * 4u, q / QE),
-                     y);
-      }
+      for (int c = 0; c < 2; ++c)
+#pragma unroll
+        for (int h = 0; h < QE; ++h) y[c * QE + h] = shoup_mul(oh[c][o * QE + h], crt_c, crt_cs, p);  // [0, 2p)
+      dsmem_st_v4_u32(HOIST ? res_r[o] : dsmem_map(res_t, o), make_uint4(y[0], y[1], y[2], y[3]));
+    }
     cluster.sync();
 
     // ---- phase 3: explicit CRT of the owned quarter, accumulate ----
+    // item m of this thread is entry m of its packed group of every prime
+    uint32_t yq[kPrimes][GRP];
+#pragma unroll
+    for (int pq = 0; pq < kPrimes; ++pq) {
+      const uint4 w = *reinterpret_cast<const uint4 *>(res + (pq * T + tau) * GRP);
+      yq[pq][0] = w.x;
+      yq[pq][1] = w.y;
+      yq[pq][2] = w.z;
+      yq[pq][3] = w.w;
+    }
 #pragma unroll
     for (int m = 0; m < ITEMS; ++m) {
       const uint32_t item = tau + m * T;
@@ -270,7 +331,7 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
       uint32_t frac = 0;
 #pragma unroll
       for (int pq = 0; pq < kPrimes; ++pq) {
-        const uint32_t y = res[(pq * 2 + c) * Q + jl];
+        const uint32_t y = yq[pq][m];
         s += static_cast<uint64_t>(y) * a.cc.pr[pq].Mp_mod64;
         frac += __umulhi(y, a.cc.pr[pq].F);  // y / p in units of 2^-27
       }
@@ -340,9 +401,11 @@ static cudaError_t launch_br_t(const BrArgs &a, cudaStream_t s) {
 template <int LOGN, bool DIG16>
 static cudaError_t launch_br_lev(const BrArgs &a, cudaStream_t s) {
   if constexpr (LOGN >= 11) {
-    // (a fixed count of 2 measured slower at N = 4096 than the runtime loop)
+    // (a compile-time level also lets phase 1 write its packed digit groups
+    // with one vector store each)
     switch (a.level) {
       case 1: return launch_br_t<LOGN, DIG16, 1>(a, s);
+      case 2: return launch_br_t<LOGN, DIG16, 2>(a, s);
       case 3: return launch_br_t<LOGN, DIG16, 3>(a, s);
       default: break;
     }

@@ -20,12 +20,14 @@
 // One CMux step is three phases separated by cluster barriers:
 //   1. each owner forms the rotated difference for its quarter (reading the
 //      rotated source coefficient from whichever CTA owns it, through
-//      distributed shared memory) and writes its gadget digits locally;
-//   2. each prime-CTA gathers all digits, runs forward NTTs two polynomials at
-//      a time, multiplies by the transform-domain BSK_i (streamed from
-//      global memory with 16-byte loads, Montgomery form), runs the two
-//      inverse NTTs and sends each owner the CRT-scaled residues of its
-//      quarter;
+//      distributed shared memory) and writes its gadget digits locally, in
+//      packed groups of four per thread;
+//   2. each prime-CTA gathers all digits (one vector DSMEM load per owner
+//      and thread), runs forward NTTs two polynomials at a time, multiplies
+//      by the transform-domain BSK_i (streamed from global memory with
+//      16-byte loads, Montgomery form), runs the two inverse NTTs and sends
+//      each owner the CRT-scaled residues of its quarter (one vector DSMEM
+//      store per owner and thread);
 //   3. each owner combines the four residues of its coefficients (explicit
 //      CRT) and adds the result to the accumulator.
 #include <cooperative_groups.h>

@@ -92,8 +92,6 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
 
   const uint32_t p = a.cc.pr[rank].p;
   const uint32_t p_inv = a.cc.pr[rank].p_inv;
-  const uint32_t crt_c = a.cc.pr[rank].crt_c;
-  const uint32_t crt_cs = a.cc.pr[rank].crt_cs;
 
   // ---- set-up: twiddles, modulus switch, accumulator ----
   for (uint32_t m = tau; m < N; m += T) tw[m] = a.tw[rank * N + m];
@@ -301,7 +299,8 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
       }
     }
     ntt_inverse<LOGN, E, 2, B::XBUF>(oh, tw, xb, tau, p);
-    // CRT-scaled residues, one packed group (component, h) per owner
+    // CRT-scaled residues (< 8p; the keys carry the CRT factor), one packed
+    // group (component, h) per owner
 #pragma unroll
     for (int o = 0; o < 4; ++o) {
       static_assert(GRP == 4, "four residues per group");
@@ -309,7 +308,7 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
 #pragma unroll
       for (int c = 0; c < 2; ++c)
 #pragma unroll
-        for (int h = 0; h < QE; ++h) y[c * QE + h] = shoup_mul(oh[c][o * QE + h], crt_c, crt_cs, p);  // [0, 2p)
+        for (int h = 0; h < QE; ++h) y[c * QE + h] = oh[c][o * QE + h];
       dsmem_st_v4_u32(HOIST ? res_r[o] : dsmem_map(res_t, o), make_uint4(y[0], y[1], y[2], y[3]));
     }
     cluster.sync();
@@ -335,9 +334,9 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
       for (int pq = 0; pq < kPrimes; ++pq) {
         const uint32_t y = yq[pq][m];
         s += static_cast<uint64_t>(y) * a.cc.pr[pq].Mp_mod64;
-        frac += __umulhi(y, a.cc.pr[pq].F);  // y / p in units of 2^-27
+        frac += __umulhi(y, a.cc.pr[pq].F);  // y / p in units of 2^-26 (y < 8p: below 2^31 in all)
       }
-      const uint32_t u = (frac + (1u << 26)) >> 27;  // round(sum y_q / p_q)
+      const uint32_t u = (frac + (1u << 25)) >> 26;  // round(sum y_q / p_q)
       acc[c * Q + jl] += s - static_cast<uint64_t>(u) * a.cc.M_mod64;
     }
     cluster.sync();

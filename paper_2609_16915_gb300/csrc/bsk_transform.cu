@@ -2,9 +2,12 @@
 // external product uses: for every GGSW row polynomial and every NTT prime,
 // the centred words (value - 2^64 when >= 2^63) reduced mod p, forward
 // negacyclic NTT (bit-reversed order, the order the blind-rotation kernel's
-// forward transforms produce), fully reduced and scaled by 2^32 mod p
-// (Montgomery form, so the kernel's Montgomery reduction of digit x key
-// products returns the plain product).
+// forward transforms produce), fully reduced and scaled by 2^32 crt_c mod p:
+// 2^32 is the Montgomery form (the kernel's Montgomery reduction of digit x
+// key products returns the plain product), crt_c = N^-1 (M/p)^-1 the factor
+// the explicit CRT needs after the inverse transform, applied here once per
+// key word instead of once per output coefficient and step (the inverse
+// transform is linear).
 //
 // Output layout [i][prime][row][component][N] uint32, so that one CTA of the
 // blind-rotation (or trace) kernel streams one contiguous block per step.
@@ -50,7 +53,7 @@ __global__ void __launch_bounds__((1 << LOGN) / 8)
 #pragma unroll
   for (int e = 0; e < 8; ++e) {
     uint32_t v = cond_sub(cond_sub(cond_sub(cond_sub(x[0][e], 8 * p), 4 * p), 2 * p), p);  // < 16p -> < p
-    v = cond_sub(shoup_mul(v, pc.r_mont, pc.r_mont_s, p), p);
+    v = cond_sub(shoup_mul(v, pc.key_scale, pc.key_scale_s, p), p);
     dst[e] = v;
   }
 }

@@ -17,11 +17,11 @@ constexpr uint32_t kPrimeList[kPrimes] = {268369921u, 268271617u, 268238849u, 26
 struct PrimeConsts {
   uint32_t p;
   uint32_t p_inv;     // p^{-1} mod 2^32 (Montgomery reduction)
-  uint32_t crt_c;     // N^{-1} * (M/p)^{-1} mod p
+  uint32_t crt_c;     // N^{-1} * (M/p)^{-1} mod p (folded into the transformed keys)
   uint32_t crt_cs;    // Shoup companion of crt_c
-  uint32_t F;         // floor(2^59 / p): fixed-point 1/p for the CRT quotient
-  uint32_t r_mont;    // 2^32 mod p
-  uint32_t r_mont_s;  // Shoup companion of r_mont
+  uint32_t F;         // floor(2^58 / p): fixed-point 1/p for the CRT quotient (inputs < 8p)
+  uint32_t key_scale;    // 2^32 crt_c mod p: Montgomery form times the CRT factor
+  uint32_t key_scale_s;  // Shoup companion of key_scale
   uint32_t pad_;
   uint64_t Mp_mod64;  // (M / p) mod 2^64
 };

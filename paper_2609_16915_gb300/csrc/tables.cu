@@ -87,9 +87,10 @@ bool build_tables(uint32_t logN, uint2 *tw_host, CrtConsts *cc) {
     const uint32_t N_inv = powmod(N, p - 2, p);
     pc.crt_c = static_cast<uint32_t>(static_cast<uint64_t>(Mq_inv) * N_inv % p);
     pc.crt_cs = shoup(pc.crt_c, p);
-    pc.F = static_cast<uint32_t>((static_cast<u128>(1) << 59) / p);
-    pc.r_mont = static_cast<uint32_t>((static_cast<uint64_t>(1) << 32) % p);
-    pc.r_mont_s = shoup(pc.r_mont, p);
+    pc.F = static_cast<uint32_t>((static_cast<u128>(1) << 58) / p);
+    const uint64_t r_mont = (static_cast<uint64_t>(1) << 32) % p;
+    pc.key_scale = static_cast<uint32_t>(r_mont * pc.crt_c % p);
+    pc.key_scale_s = shoup(pc.key_scale, p);
     pc.pad_ = 0;
     pc.Mp_mod64 = static_cast<uint64_t>(Mq);
   }

@@ -70,8 +70,6 @@ __global__ void __launch_bounds__(TrShape<LOGN>::T) trace_kernel(const TraceArgs
 
   const uint32_t p = a.cc.pr[rank].p;
   const uint32_t p_inv = a.cc.pr[rank].p_inv;
-  const uint32_t crt_c = a.cc.pr[rank].crt_c;
-  const uint32_t crt_cs = a.cc.pr[rank].crt_cs;
 
   for (uint32_t m = tau; m < N; m += T) tw[m] = a.tw[rank * N + m];
   const uint64_t *gin = a.glwe_in + static_cast<size_t>(ct) * 2 * N;
@@ -178,7 +176,7 @@ __global__ void __launch_bounds__(TrShape<LOGN>::T) trace_kernel(const TraceArgs
     for (int c = 0; c < 2; ++c)
 #pragma unroll
       for (int q = 0; q < E; ++q) {
-        const uint32_t y = shoup_mul(oh[c][q], crt_c, crt_cs, p);
+        const uint32_t y = oh[c][q];  // < 8p, CRT-scaled through the keys
         dsmem_st_u32(dsmem_map(res_s + ((rank * 2 + c) * Q + tau + (q % QE) * T) * 4u, q / QE), y);
       }
     cluster.sync();
@@ -196,7 +194,7 @@ __global__ void __launch_bounds__(TrShape<LOGN>::T) trace_kernel(const TraceArgs
         sum += static_cast<uint64_t>(y) * a.cc.pr[pq].Mp_mod64;
         frac += __umulhi(y, a.cc.pr[pq].F);
       }
-      const uint32_t u = (frac + (1u << 26)) >> 27;
+      const uint32_t u = (frac + (1u << 25)) >> 26;
       const uint64_t X = sum - static_cast<uint64_t>(u) * a.cc.M_mod64;
       if (PTMUL)
         acc[c * Q + jl] = X + ((c == 1 && a.plain_add) ? a.plain_add[rank * Q + jl] : 0ull);

@@ -94,8 +94,12 @@ typedef struct {
  * scratch for p->max_batch ciphertexts.  *out receives the context (NULL on
  * error).  UNSUPPORTED_PARAMS also when the exact external product would
  * not fit the four NTT primes: log2((k+1) l N 2^(beta-1) 2^63) + 1 must not
- * exceed 111 (their product is about 2^111.99).  Errors: INVALID_ARG (NULL),
- * UNSUPPORTED_PARAMS, CUDA, OOM. */
+ * exceed 111 (their product is about 2^111.99); and when one blind-rotation
+ * CTA (a quarter of the ring) does not fit the device's shared memory per
+ * block: 20N + 4.5N per exchange buffer (two for N <= 1024, else one) +
+ * l N x {1 for beta <= 16 | 2} + 2(n+1) bytes, which on a 227 KB device
+ * admits, at N = 8192, l <= 3 with beta <= 16 (n <= 3583) or l = 1 with
+ * beta > 16.  Errors: INVALID_ARG (NULL), UNSUPPORTED_PARAMS, CUDA, OOM. */
 int rosetta_params_init(rosetta_ctx **out, const rosetta_params *p, int cuda_device);
 
 /* Upload the raw bootstrapping key (layout above, n_words =

@@ -486,3 +486,21 @@ def test_plaintext_mul_scales_the_phase():
             t = i + j
             want[t % N] += int(P[i]) * int(m[j]) * (-1 if t >= N else 1)
     assert [int(x) for x in ph] == [x % Q for x in want]
+
+
+@pytest.mark.parametrize("N,base_log,level", [(64, 28, 2), (128, 16, 4), (64, 21, 3), (256, 9, 7)])
+@pytest.mark.parametrize("sign", [+1, -1])
+def test_cmux_at_the_largest_magnitude_closed_form(N, base_log, level, sign):
+    """One CMux with a~ = N on a GLWE of constant C/2: every digit of the
+    CMux input is -B/2 (closed form of the balanced decomposition), so the
+    rotated GLWE is C/2 plus -B/2 times the negacyclic running sums of the
+    key words -- every coefficient known without the oracle's arithmetic."""
+    from tests import extreme_util as X
+    p = W.Params("extreme", n=2, k=1, N=N, pbs_base_log=base_log, pbs_level=level, ks_base_log=4, ks_level=4,
+                 msg_bits=3, lwe_sigma_log2=40, glwe_sigma_log2=20, lut=("square_mod",), msg=("uniform",),
+                 batch=1, seed=1)
+    bsk, lwe, glwe, C = X.case(p, sign, seed=N + level)
+    got = O.blind_rotate_glwe_batch(p, bsk, lwe, glwe)
+    want, peak = X.expected(p, bsk, C)
+    assert peak > 1 << (62 + base_log)
+    assert [[int(w) for w in row] for row in got[0]] == want

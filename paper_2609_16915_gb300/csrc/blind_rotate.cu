@@ -329,14 +329,14 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
       const uint32_t item = tau + m * T;
       const uint32_t c = item / Q, jl = item % Q;
       uint64_t s = 0;
-      uint32_t frac = 0;
+      uint32_t ysum = 0;
 #pragma unroll
       for (int pq = 0; pq < kPrimes; ++pq) {
         const uint32_t y = yq[pq][m];
         s += static_cast<uint64_t>(y) * a.cc.pr[pq].Mp_mod64;
-        frac += __umulhi(y, a.cc.pr[pq].F);  // y / p in units of 2^-26 (y < 8p: below 2^31 in all)
+        ysum += y >> 2;  // y < 8p < 2^31: the sum stays below 2^31
       }
-      const uint32_t u = (frac + (1u << 25)) >> 26;  // round(sum y_q / p_q)
+      const uint32_t u = crt_quotient(ysum);
       acc[c * Q + jl] += s - static_cast<uint64_t>(u) * a.cc.M_mod64;
     }
     cluster.sync();

@@ -6,7 +6,7 @@
 
 namespace rosetta {
 
-// Four NTT primes p = c * 2^14 + 1 in (2^27, 2^28): 2N | p - 1 for every
+// Four NTT primes p = c * 2^14 + 1 in (2^28 - 2^18, 2^28): 2N | p - 1 for every
 // N <= 8192, 16p < 2^32 leaves room for lazily reduced residues, and their
 // product M > 2^111.99 exceeds twice the largest exact integer value of an
 // external-product coefficient, (k+1) l N 2^(beta-1) 2^63, for every
@@ -19,10 +19,8 @@ struct PrimeConsts {
   uint32_t p_inv;     // p^{-1} mod 2^32 (Montgomery reduction)
   uint32_t crt_c;     // N^{-1} * (M/p)^{-1} mod p (folded into the transformed keys)
   uint32_t crt_cs;    // Shoup companion of crt_c
-  uint32_t F;         // floor(2^58 / p): fixed-point 1/p for the CRT quotient (inputs < 8p)
   uint32_t key_scale;    // 2^32 crt_c mod p: Montgomery form times the CRT factor
   uint32_t key_scale_s;  // Shoup companion of key_scale
-  uint32_t pad_;
   uint64_t Mp_mod64;  // (M / p) mod 2^64
 };
 

@@ -25,6 +25,15 @@ __device__ __forceinline__ uint32_t redc(uint64_t T, uint32_t p, uint32_t p_inv)
   return static_cast<uint32_t>(T >> 32) - t + p;
 }
 
+// Quotient of the explicit CRT, round(sum_q y_q / p_q), from ysum = sum_q
+// (y_q >> 2) with every y_q < 8 p_q.  The primes lie in (2^28 - 2^18, 2^28),
+// so y / 2^28 undershoots y / p by less than 8 (2^28 - p) / 2^28 < 2^-7 per
+// prime (the shift adds under 2^-26); the four together by less than 2^-5.
+// The exact sum is an integer plus X / M with |X| <= 2^110 < M / 3.99 (the
+// bound every accepted parameter set meets), so the estimate stays within
+// 0.29 of that integer and rounds to it.
+__device__ __forceinline__ uint32_t crt_quotient(uint32_t ysum) { return (ysum + (1u << 25)) >> 26; }
+
 // x in [0, 2b) -> [0, b) for a bound b: one subtraction when x >= b.
 __device__ __forceinline__ uint32_t cond_sub(uint32_t x, uint32_t b) {
   return min(x, x - b);

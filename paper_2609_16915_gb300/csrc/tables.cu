@@ -67,7 +67,9 @@ bool build_tables(uint32_t logN, uint2 *tw_host, CrtConsts *cc) {
   cc->M_mod64 = static_cast<uint64_t>(M);
   for (int q = 0; q < kPrimes; ++q) {
     const uint32_t p = kPrimeList[q];
-    if (!is_prime(p) || (p - 1) % (2 * N) != 0 || p >= (1u << 28) || p <= (1u << 27)) return false;
+    // (2^28 - 2^18, 2^28): lazy residues up to 16p fit 32 bits, and the CRT
+    // quotient may use 2^28 in place of p
+    if (!is_prime(p) || (p - 1) % (2 * N) != 0 || p >= (1u << 28) || p <= (1u << 28) - (1u << 18)) return false;
     const uint32_t g = generator(p);
     if (!g) return false;
     const uint32_t psi = powmod(g, (p - 1) / (2 * N), p);  // primitive 2N-th root of unity
@@ -87,11 +89,9 @@ bool build_tables(uint32_t logN, uint2 *tw_host, CrtConsts *cc) {
     const uint32_t N_inv = powmod(N, p - 2, p);
     pc.crt_c = static_cast<uint32_t>(static_cast<uint64_t>(Mq_inv) * N_inv % p);
     pc.crt_cs = shoup(pc.crt_c, p);
-    pc.F = static_cast<uint32_t>((static_cast<u128>(1) << 58) / p);
     const uint64_t r_mont = (static_cast<uint64_t>(1) << 32) % p;
     pc.key_scale = static_cast<uint32_t>(r_mont * pc.crt_c % p);
     pc.key_scale_s = shoup(pc.key_scale, p);
-    pc.pad_ = 0;
     pc.Mp_mod64 = static_cast<uint64_t>(Mq);
   }
   return true;

@@ -187,14 +187,14 @@ __global__ void __launch_bounds__(TrShape<LOGN>::T) trace_kernel(const TraceArgs
       const uint32_t item = tau + m * T;
       const uint32_t c = item / Q, jl = item % Q;
       uint64_t sum = 0;
-      uint32_t frac = 0;
+      uint32_t ysum = 0;
 #pragma unroll
       for (int pq = 0; pq < kPrimes; ++pq) {
         const uint32_t y = res[(pq * 2 + c) * Q + jl];
         sum += static_cast<uint64_t>(y) * a.cc.pr[pq].Mp_mod64;
-        frac += __umulhi(y, a.cc.pr[pq].F);
+        ysum += y >> 2;
       }
-      const uint32_t u = (frac + (1u << 25)) >> 26;
+      const uint32_t u = crt_quotient(ysum);
       const uint64_t X = sum - static_cast<uint64_t>(u) * a.cc.M_mod64;
       if (PTMUL)
         acc[c * Q + jl] = X + ((c == 1 && a.plain_add) ? a.plain_add[rank * Q + jl] : 0ull);

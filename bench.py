@@ -400,7 +400,7 @@ def main():
     ap.add_argument("--config", default="standard", choices=sorted(W.CONFIGS))
     ap.add_argument("--batch", type=int, default=0, help="override the workload's batch")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--cpu-sample", type=int, default=0, help="oracle sample size (default: host cores)")
+    ap.add_argument("--cpu-sample", type=int, default=0, help="oracle sample size (default: three per host core)")
     ap.add_argument("--path", default="pbs", choices=["pbs", "lookup", "multi_lut"])
     args = ap.parse_args()
     p = W.CONFIGS[args.config]
@@ -551,7 +551,7 @@ def main():
         import oracle as O
         O.build()
         cores = O.default_threads()
-        sample = args.cpu_sample or cores
+        sample = args.cpu_sample or 3 * cores  # three ciphertexts per core: about 13 s on 16 Grace cores
         r, dt, t = oracle_pbs_rate(p, sample, threads=cores)
         line["cpu_baseline"] = {"value": r, "unit": UNIT, "cores": t, "kind": "oracle",
                                 "sample": f"{sample} ciphertexts of the workload, uniform-word keys, {dt:.1f} s"}

@@ -30,6 +30,11 @@ def _lib():
 _KEYS = {}
 
 
+def torch_device_count():
+    import torch
+    return torch.cuda.device_count()
+
+
 def real_keys(name):
     if name not in _KEYS:
         p = W.CONFIGS[name]
@@ -290,6 +295,15 @@ def test_error_codes():
     st = L.rosetta_upload_bsk(ctx._h, G.to_dev(keys.bsk).data_ptr(), keys.bsk.size - 1, 1, None)
     assert st == -1                               # wrong key size
     ctx.sync_status()
+    small = G.make_ctx(p, keys.bsk, keys.ksk, max_batch=2)
+    with pytest.raises(R.RosettaError) as e:      # batch above the context's max_batch
+        small.pbs_batch(lwe, lut, out)
+    assert e.value.status == -1
+    got = G.gpu_pbs(small, p, W.uniform_ciphertexts(p, 2), W.lut_torus(p))
+    assert got.shape == (2, p.n + 1)
+    with pytest.raises(R.RosettaError) as e:      # no such device
+        R.Context(p, device=torch_device_count() + 3)
+    assert e.value.status == -4
 
 
 def test_c_client_bootstraps_like_the_oracle(tmp_path):

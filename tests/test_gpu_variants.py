@@ -91,3 +91,30 @@ def test_external_product_at_its_largest_magnitude(N, base_log, level, sign):
     want, peak = X.expected(p, bsk, C)
     assert peak > 1 << 100
     assert [[int(w) for w in row] for row in got[0]] == want
+
+
+@pytest.mark.parametrize("n", [1, 65535])
+def test_lwe_dimension_extremes(n):
+    """The smallest and the largest LWE dimension the library accepts (the
+    a~_i are kept in shared memory as 16-bit words); nonzero masks at the
+    first and the last index, so the first and the last CMux step both run."""
+    p = W.Params(f"n{n}", n=n, k=1, N=256, pbs_base_log=16, pbs_level=1, ks_base_log=4, ks_level=4, msg_bits=3,
+                 lwe_sigma_log2=40, glwe_sigma_log2=20, lut=("square_mod",), msg=("uniform",), batch=2, seed=n)
+    bsk, ksk = W.uniform_keys(p)
+    g = np.random.default_rng(n)
+    lwe = np.zeros((2, n + 1), np.uint64)
+    for b in range(2):
+        for i in {0, n - 1, n // 2}:
+            lwe[b, i] = g.integers(0, 2**64, dtype=np.uint64, endpoint=False)
+        lwe[b, n] = g.integers(0, 2**64, dtype=np.uint64, endpoint=False)
+    lut = W.lut_torus(p)
+    ctx = G.make_ctx(p, bsk, ksk)
+    big = G.gpu_br_extract(ctx, p, lwe, lut)
+    want_big = O.blind_rotate_extract_batch(p, bsk, lwe, lut)
+    assert np.array_equal(big, want_big)
+    assert np.array_equal(G.gpu_pbs(ctx, p, lwe, lut), O.keyswitch_batch(p, ksk, want_big))
+    import paper_2609_16915_gb300 as R
+    if n == 65535:
+        with pytest.raises(R.RosettaError) as e:
+            R.Context(W.Params(**{**p.__dict__, "n": 65536}), device=0)
+        assert e.value.status == -2

@@ -105,10 +105,15 @@ __device__ __forceinline__ void gs_bfly(uint32_t &X, uint32_t &Y, uint2 w, uint3
 // the very first inverse stage (LAST pass), whose inputs are all below 4p.
 template <bool LAST, int H, int U>
 __host__ __device__ constexpr bool inv_corrects(int q) {
-  if (U >= H - 1) return !LAST;
-  if (((q >> (H - U - 2)) & 1) != 0) return false;
-  if (U + 2 <= H - 1 && ((q >> (H - U - 3)) & 1) == 1) return false;
-  return true;
+  if constexpr (U >= H - 1) {
+    return !LAST;
+  } else {
+    if (((q >> (H - U - 2)) & 1) != 0) return false;
+    if constexpr (U + 2 <= H - 1) {
+      if (((q >> (H - U - 3)) & 1) == 1) return false;
+    }
+    return true;
+  }
 }
 
 // Load CNT (a power of two) consecutive twiddle pairs starting at an index

@@ -95,3 +95,20 @@ def build_c_client(out_path):
 def test_c_client_compiles_and_links(lib, tmp_path):
     """The header is plain C and the library links from C without CUDA headers."""
     assert os.path.exists(build_c_client(str(tmp_path / "c_abi_demo")))
+
+
+def declared_arity():
+    """Parameter count of every prototype in the header."""
+    text = re.sub(r"/\*.*?\*/", "", open(HEADER).read(), flags=re.S)
+    out = {}
+    for name, params in re.findall(r"\b(rosetta_[a-z_]+)\s*\(([^)]*)\)\s*;", text):
+        params = params.strip()
+        out[name] = 0 if params in ("", "void") else params.count(",") + 1
+    return out
+
+
+def test_binding_argument_counts_match_the_header(lib):
+    arity = declared_arity()
+    assert set(arity) == set(declared_functions())
+    for name, n in arity.items():
+        assert len(getattr(lib, name).argtypes) == n, name

@@ -45,6 +45,26 @@ def test_multi_lut_bitexact_and_decrypts():
     assert np.array_equal(keys.decrypt(got), want_codes)
 
 
+def test_multi_lut_full_batch_sampled():
+    """The benchmark's many-LUT launch: standard set, 4096 ciphertexts, four
+    LUTs round-robin; sparse-mask inputs at seeded positions are checked
+    word for word, the rest are dense uniform words."""
+    p = W.CONFIGS["standard"]
+    bsk, ksk = W.uniform_keys(p, seed=61)
+    codes = W.lut_codes(p)
+    luts = np.stack([W.lut_torus(p, np.roll(codes, r)) for r in range(4)])
+    idx = np.arange(p.batch) % 4
+    lwe = W.uniform_ciphertexts(p, p.batch, sub=62)
+    pos = np.array([0, 1, 2, 3, p.batch - 1])
+    lwe[pos] = G.sparse_lwe(p, len(pos), 2, seed=63)
+    ctx = G.make_ctx(p, bsk, ksk, max_batch=p.batch)
+    out = G.empty_dev(p.batch, p.n + 1)
+    ctx.pbs_batch_multi_lut(G.to_dev(lwe), G.to_dev(luts), _index_dev(idx), out)
+    ctx.sync_status()
+    got = G.to_host(out)
+    assert np.array_equal(got[pos], O.pbs_batch_multi_lut(p, bsk, ksk, lwe[pos], luts, idx[pos]))
+
+
 def test_multi_lut_bad_index_is_reported_not_followed():
     import paper_2609_16915_gb300 as R
     p = W.CONFIGS["tiny"]
@@ -310,6 +330,31 @@ def test_lookup_bitexact_standard_ring():
     ctx.segmented_lookup_batch(G.to_dev(glwe), G.to_dev(lwe), out)
     ctx.sync_status()
     assert np.array_equal(G.to_host(out), O.segmented_lookup_batch(p, bsk, ksk, tk, 16, 4, glwe, lwe, *tables))
+
+
+def test_lookup_full_batch_sampled():
+    """The benchmark's lookup launch: standard ring, 1024 ciphertexts, four
+    segments, trace gadget 2^16 x 4; two seeded positions (sparse segment
+    index ciphertexts, for the oracle's cost) are checked word for word."""
+    p = W.CONFIGS["standard"]
+    g = np.random.default_rng(70)
+    batch, n_seg = 1024, 4
+    bsk, ksk = W.uniform_keys(p, seed=71)
+    tk = W.uniform_u64((p.N.bit_length() - 1, 4, 2, p.N), W.rng(p.seed, "sample", 72))
+    tables = (g.integers(-2**40, 2**40, size=p.N, dtype=np.int64), W.uniform_u64((p.N,), W.rng(p.seed, "sample", 73)),
+              g.integers(-2**40, 2**40, size=(n_seg, p.N), dtype=np.int64),
+              W.uniform_u64((n_seg, p.N), W.rng(p.seed, "sample", 74)))
+    glwe = W.uniform_u64((batch, 2, p.N), W.rng(p.seed, "sample", 75))
+    lwe = W.uniform_ciphertexts(p, batch, sub=76)
+    pos = np.array([0, batch - 1])
+    lwe[pos] = G.sparse_lwe(p, len(pos), 3, seed=77)
+    ctx = _lookup_ctx(p, bsk, ksk, tk, 16, 4, tables)
+    out = G.empty_dev(batch, 2, p.N)
+    ctx.segmented_lookup_batch(G.to_dev(glwe), G.to_dev(lwe), out)
+    ctx.sync_status()
+    got = G.to_host(out)
+    want = O.segmented_lookup_batch(p, bsk, ksk, tk, 16, 4, glwe[pos], lwe[pos], *tables)
+    assert np.array_equal(got[pos], want)
 
 
 def test_lookup_argument_checks():

@@ -255,11 +255,16 @@ int rosetta_segmented_lookup_batch(rosetta_ctx *ctx, const uint64_t *glwe_x, con
  * library (held on every device that loads it until exit) instead of a
  * buffer grown with cudaMallocAsync, so batch * (kN+1) must not exceed
  * 2^21 words (1023 ciphertexts at N = 2048, 255 at N = 8192); larger
- * batches return INVALID_ARG.  lwe_in, lut and lwe_out must be device
- * memory (no host staging).  The first call on a device looks up the
- * array's device address; make it before any stream capture.  All calls on a
- * device share the array: calls whose work overlaps on the GPU race and must
- * be serialised by the caller.  Errors: INVALID_ARG, KEYS_MISSING, CUDA. */
+ * batches return INVALID_ARG, and so do batches above the context's
+ * max_batch, as in rosetta_pbs_batch.  lwe_in, lut and lwe_out must be
+ * device memory (no host staging).  Every call looks up the array's device
+ * address in the current CUDA context; the first call on a device (and the
+ * first after a device reset) loads the library's device code: make it
+ * before any stream capture.  The key switch is the CUDA-core kernel at
+ * every batch size, because the tensor-core one needs digit tiles in
+ * allocated memory (same words).  All calls on a device share the array:
+ * calls whose work overlaps on the GPU race and must be serialised by the
+ * caller.  Errors: INVALID_ARG, KEYS_MISSING, CUDA. */
 int rosetta_pbs_batch_noalloc(rosetta_ctx *ctx, const uint64_t *lwe_in, uint32_t batch,
                               const uint64_t *lut, uint64_t *lwe_out, void *stream);
 

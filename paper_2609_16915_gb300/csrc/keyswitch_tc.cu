@@ -27,8 +27,10 @@
 // filled by cp.async.bulk, one thread issuing tcgen05.mma (M = 128, N = 256,
 // K = 16, four per step) into 256 columns of tensor memory, and four warps
 // reading their 32 lanes back with tcgen05.ld for the recombination.  Every
-// wait on an mbarrier gives up after about two seconds, sets the error flag,
-// drains what it issued and frees the tensor memory.
+// wait on an mbarrier gives up after about two seconds and sets the error
+// flag; the CTA then skips its epilogue, waits (again bounded) for the copies
+// it issued, and frees the tensor memory only when nothing it issued can
+// still be in flight.
 #include <stdint.h>
 
 #include "dsmem.cuh"
@@ -193,6 +195,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1) ks_tc_kernel(const KsTcArgs a) 
   extern __shared__ __align__(1024) unsigned char smem[];
   __shared__ __align__(8) uint64_t bars[2 * TC_STAGES + 1];  // full[s], empty[s], done
   __shared__ uint32_t tmem_slot;
+  // set when a wait gave up: s_fail, a copy or an MMA slot never completed
+  // (the accumulators are partial); s_unsafe, copies or MMAs this CTA issued
+  // may still be in flight
+  __shared__ uint32_t s_fail, s_unsafe;
   const uint32_t nt = blockIdx.x, mt = blockIdx.y;
   const uint32_t warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const uint32_t base = smem_addr(smem);
@@ -208,6 +214,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1) ks_tc_kernel(const KsTcArgs a) 
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
   if (threadIdx.x == 0) {
+    s_fail = 0u;
+    s_unsafe = 0u;
     for (uint32_t s = 0; s < 2 * TC_STAGES + 1; ++s) mbar_init(bar0 + 8u * s, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -255,16 +263,26 @@ __global__ void __launch_bounds__(TC_THREADS, 1) ks_tc_kernel(const KsTcArgs a) 
       mma_commit(done);
       if (!ok) {
         atomicExch(a.err_flag, 2u);
+        s_fail = 1u;
         // let the copies already issued land before the shared memory is released
-        for (uint32_t k = consumed; k < issued; ++k) mbar_wait(full(k % TC_STAGES), (k / TC_STAGES) & 1u);
+        bool drained = true;
+        for (uint32_t k = consumed; k < issued; ++k)
+          drained = mbar_wait(full(k % TC_STAGES), (k / TC_STAGES) & 1u) && drained;
+        if (!drained) s_unsafe = 1u;
       }
     }
     __syncwarp();
   }
   const bool fin = __all_sync(0xffffffffu, mbar_wait(done, 0));  // warp-uniform for tcgen05.ld
+  if (!fin && lane == 0) {
+    atomicExch(a.err_flag, 2u);
+    s_unsafe = 1u;  // the MMAs may still be writing tensor memory
+  }
+  __syncthreads();
+  const bool unsafe = s_unsafe != 0u, partial = s_fail != 0u;
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 
-  if (fin) {
+  if (!unsafe && !partial) {
     // epilogue: lane = ciphertext row of this warp's quarter of tensor memory
     const uint32_t row = warp * 32 + lane;
     const uint32_t b = mt * TC_M + row;
@@ -288,12 +306,14 @@ __global__ void __launch_bounds__(TC_THREADS, 1) ks_tc_kernel(const KsTcArgs a) 
         if (b < a.batch && j < n1) a.out[static_cast<size_t>(b) * n1 + j] = (j == a.n ? body : 0ull) - s;
       }
     }
-  } else if (threadIdx.x == 0) {
-    atomicExch(a.err_flag, 2u);
   }
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
   __syncthreads();
-  if (warp == 0)
+  // After a wait that gave up with work still in flight nothing is safe: the
+  // tensor memory is left allocated rather than handed to another CTA while
+  // an MMA may still write it, the outputs are not written, and the error
+  // flag reports TIMEOUT.  The CUDA context must then be destroyed.
+  if (warp == 0 && !unsafe)
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TMEM_COLS) : "memory");
 }
 

@@ -14,16 +14,23 @@
 //
 // The array is a file-scope __device__ variable: every GPU that loads the
 // library holds it until the process exits, and all calls on a device share
-// it.  Host code cannot use its name as a device address, so the address is
-// looked up once per device with cudaGetSymbolAddress, on the first call
-// made on that device (make that first call before any stream capture).
-// Calls whose work overlaps on the GPU (for example on two streams) race on
-// the array and must be serialised by the caller.  Nothing in it has to start
-// at zero: the blind-rotation kernel writes all kN+1 words of every
-// ciphertext slot it uses before the key switch reads them.
+// it.  Host code cannot use its name as a device address, so every call looks
+// the address up with cudaGetSymbolAddress on the context's device.  The
+// lookup is a host-side table read once the library's device code is loaded
+// in the current CUDA context; it is not cached across calls because a
+// context that is torn down (cudaDeviceReset) and re-created loads the
+// module again at a different address.  The first call on a device, and the
+// first after such a reset, loads the module: make it before any stream
+// capture.  Calls whose work overlaps on the GPU (for example on two
+// streams) race on the array and must be serialised by the caller.  Nothing
+// in it has to start at zero: the blind-rotation kernel writes all kN+1
+// words of every ciphertext slot it uses before the key switch reads them.
+//
+// The key switch is the CUDA-core kernel (keyswitch_kernel) at every batch
+// size: the tensor-core kernel that rosetta_pbs_batch uses from 256
+// ciphertexts on needs digit tiles in a buffer the library allocates.  Both
+// give the same words.
 #include <cuda_runtime.h>
-
-#include <mutex>
 
 #include "context.h"
 #include "internal.h"
@@ -36,21 +43,13 @@ namespace {
 constexpr size_t kNoallocScratchWords = size_t(2) << 20;
 static __device__ __align__(256) uint64_t g_noalloc_scratch[kNoallocScratchWords];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_noalloc_mu;
-uint64_t *g_noalloc_addr[kMaxDevices] = {};
-
-// Device address of g_noalloc_scratch on device `dev` (which must be current).
-int noalloc_scratch(int dev, uint64_t **out) {
-  if (dev < 0 || dev >= kMaxDevices) return ROSETTA_ERR_INVALID_ARG;
-  std::lock_guard<std::mutex> lock(g_noalloc_mu);
-  if (!g_noalloc_addr[dev]) {
-    void *p = nullptr;
-    const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-    if (e != cudaSuccess || !p) return ROSETTA_ERR_CUDA;
-    g_noalloc_addr[dev] = static_cast<uint64_t *>(p);
-  }
-  *out = g_noalloc_addr[dev];
+// Device address of g_noalloc_scratch in the current context (the caller
+// has made the context's device current).
+int noalloc_scratch(uint64_t **out) {
+  void *p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+  if (e != cudaSuccess || !p) return ROSETTA_ERR_CUDA;
+  *out = static_cast<uint64_t *>(p);
   return ROSETTA_OK;
 }
 
@@ -74,6 +73,7 @@ extern "C" int rosetta_pbs_batch_noalloc(rosetta_ctx *c, const uint64_t *lwe_in,
   const size_t kN = static_cast<size_t>(c->prm.glwe_dim) * c->prm.poly_size;
   const size_t n1 = c->prm.lwe_dim + 1;
   if (static_cast<size_t>(batch) * (kN + 1) > kNoallocScratchWords) return ROSETTA_ERR_INVALID_ARG;
+  if (c->prm.max_batch && batch > c->prm.max_batch) return ROSETTA_ERR_INVALID_ARG;  // as rosetta_pbs_batch
   const uintptr_t mis = (reinterpret_cast<uintptr_t>(lwe_in) | reinterpret_cast<uintptr_t>(lut) |
                          reinterpret_cast<uintptr_t>(lwe_out)) & 7u;
   if (mis) return ROSETTA_ERR_INVALID_ARG;
@@ -84,7 +84,7 @@ extern "C" int rosetta_pbs_batch_noalloc(rosetta_ctx *c, const uint64_t *lwe_in,
   // no staging of host memory here: every buffer must already be on the device
   if (!on_device(lwe_in) || !on_device(lut) || !on_device(lwe_out)) return ROSETTA_ERR_INVALID_ARG;
   uint64_t *big = nullptr;
-  const int st = noalloc_scratch(c->device, &big);
+  const int st = noalloc_scratch(&big);
   if (st != ROSETTA_OK) return st;
   const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
 

@@ -10,6 +10,7 @@ import ctypes
 import numpy as np
 import pytest
 
+import oracle as O
 import workload as W
 
 pytestmark = pytest.mark.gpu
@@ -39,17 +40,27 @@ def _call_noalloc(R, ctx, lwe, lut, out):
 
 def test_noalloc_matches_pbs_batch_twice_in_a_row(setup):
     R, G, p, ctx = setup
-    lut = G.to_dev(W.lut_torus(p))
-    first = G.to_dev(W.uniform_ciphertexts(p, 300, sub=31))
+    lut_h = W.lut_torus(p)
+    lut = G.to_dev(lut_h)
+    first_h = W.uniform_ciphertexts(p, 300, sub=31)
+    first_h[[0, 299]] = G.sparse_lwe(p, 2, 3, seed=33)          # short chains at the ends
+    first = G.to_dev(first_h)
     second = G.to_dev(W.uniform_ciphertexts(p, 77, sub=32))   # smaller: stale words from call 1 remain
-    for lwe in (first, second):
+    for call, lwe in enumerate((first, second)):
         want = G.empty_dev(lwe.shape[0], p.n + 1)
         ctx.pbs_batch(lwe, lut, want, stream=0)
         ctx.sync_status(stream=0)
         got = G.empty_dev(lwe.shape[0], p.n + 1)
         assert _call_noalloc(R, ctx, lwe, lut, got) == 0
         ctx.sync_status(stream=0)
-        assert np.array_equal(G.to_host(got), G.to_host(want))
+        got_h = G.to_host(got)
+        assert np.array_equal(got_h, G.to_host(want))
+        if call == 0:
+            # and against the CPU oracle at sampled positions (150: a dense
+            # chain of all n CMux steps)
+            pos = np.array([0, 150, 299])
+            bsk, ksk = W.uniform_keys(p, seed=21)
+            assert np.array_equal(got_h[pos], O.pbs_batch(p, bsk, ksk, first_h[pos], lut_h))
 
 
 def test_noalloc_rejects_oversize_and_host_buffers(setup):
@@ -67,3 +78,10 @@ def test_noalloc_rejects_oversize_and_host_buffers(setup):
     ok_in = big[:limit]
     assert _call_noalloc(R, ctx, ok_in, lut, out[:limit]) == 0
     ctx.sync_status(stream=0)
+    # a context's max_batch binds this entry point as it binds rosetta_pbs_batch
+    bsk, ksk = W.uniform_keys(p, seed=21)
+    small = G.make_ctx(p, bsk, ksk, max_batch=2)
+    assert _call_noalloc(R, small, big[:3], lut, out[:3]) == -1
+    assert _call_noalloc(R, small, big[:2], lut, out[:2]) == 0
+    small.sync_status(stream=0)
+    small.close()

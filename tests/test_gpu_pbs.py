@@ -199,17 +199,6 @@ def test_large_configs_full_batch_sparse_sample(name):
     assert np.array_equal(got[pos], want)
 
 
-def test_gpt2_mlp_real_keys_decrypt():
-    p = W.CONFIGS["gpt2_mlp"]
-    keys = real_keys("gpt2_mlp")
-    cd = W.cipher_draws(p, p.batch, sub=6)
-    lwe = keys.encrypt(cd)
-    ctx = G.make_ctx(p, keys.bsk, keys.ksk, max_batch=p.batch)
-    got = G.gpu_pbs(ctx, p, lwe, W.lut_torus(p))
-    fails = int(np.sum(keys.decrypt(got) != W.lut_codes(p)[cd.codes]))
-    assert fails == 0
-
-
 # ------------------------------------------------------------------ edge cases
 
 def test_edge_inputs_match_oracle():

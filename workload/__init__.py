@@ -11,9 +11,13 @@ ciphertext; Evaluation, "Experimental Setup": LUT precision, ranges).  The
 torus is Z_{2^64}; every ciphertext word is a uint64.
 
 Randomness: numpy's PCG64 bit generator (O'Neill 2014) seeded through a
-SeedSequence([master_seed, purpose]).  Uniform words are raw 64-bit outputs;
-Gaussian noise is numpy's standard normal scaled by 2^sigma_log2 and rounded
-to the nearest integer, stored as two's complement.
+SeedSequence([master_seed, purpose]); only its raw 64-bit outputs are used,
+whose stream numpy keeps fixed across versions and platforms.  Uniform words
+are raw outputs.  Normal variates are the Irwin-Hall sum of twelve uniforms
+minus six (mean 0, variance 1, tails cut at 6 sigma), formed in integer
+arithmetic from the top 53 bits of twelve raw outputs, so every draw is the
+same on every host; Gaussian noise is that variate times 2^sigma_log2,
+rounded half up to an integer, stored as two's complement.
 """
 
 from __future__ import annotations
@@ -135,11 +139,32 @@ def binary_u64(shape, g: np.random.Generator) -> np.ndarray:
     return (uniform_u64(shape, g) >> np.uint64(63)).astype(np.uint64)
 
 
+_IH_TERMS = 12      # uniforms per normal variate
+_IH_BITS = 53       # bits kept of each raw output
+
+
+def normal_fixed(count: int, g: np.random.Generator) -> np.ndarray:
+    """Approximately standard normal variates as exact integers z * 2^53:
+    the sum of twelve uniform 53-bit integers minus 6 * 2^53 (Irwin-Hall:
+    mean 0, variance 1, |z| < 6), int64."""
+    u = (g.bit_generator.random_raw(_IH_TERMS * count).astype(np.uint64) >> np.uint64(64 - _IH_BITS)).astype(np.int64)
+    return u.reshape(count, _IH_TERMS).sum(axis=1) - np.int64(6 << _IH_BITS)
+
+
+def standard_normal(count: int, g: np.random.Generator) -> np.ndarray:
+    """The same variates as float64 (z * 2^53 rounded to 53 bits, then
+    scaled by 2^-53: IEEE arithmetic, identical on every host)."""
+    return normal_fixed(count, g).astype(np.float64) * (2.0 ** -_IH_BITS)
+
+
 def gaussian_u64(shape, sigma_log2: int, g: np.random.Generator) -> np.ndarray:
-    """round(2^sigma_log2 * z), z ~ N(0,1), as two's-complement uint64."""
-    z = g.standard_normal(int(np.prod(shape)))
-    v = np.rint(z * (2.0 ** sigma_log2)).astype(np.int64)
-    return v.view(np.uint64).reshape(shape)
+    """round(2^sigma_log2 * z) (ties up), z from normal_fixed, as
+    two's-complement uint64; exact integer arithmetic (sigma_log2 < 53)."""
+    assert 0 <= sigma_log2 < _IH_BITS
+    zf = normal_fixed(int(np.prod(shape)), g)
+    sh = _IH_BITS - sigma_log2
+    v = (zf + np.int64(1 << (sh - 1))) >> np.int64(sh)      # arithmetic shift: floor
+    return v.astype(np.int64).view(np.uint64).reshape(shape)
 
 
 # --------------------------------------------------------------------------
@@ -196,7 +221,7 @@ def message_codes(params: Params, count: int, g: np.random.Generator) -> np.ndar
     if params.msg[0] == "uniform":
         return (uniform_u64((count,), g) % np.uint64(size)).astype(np.int64)
     _, std, lo, hi = params.msg
-    x = np.clip(g.standard_normal(count) * std, lo, hi)
+    x = np.clip(standard_normal(count, g) * std, lo, hi)
     m = np.floor((x - lo) / (hi - lo) * size).astype(np.int64)
     return np.clip(m, 0, size - 1)
 

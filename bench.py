@@ -13,7 +13,9 @@ the host cores instead (the reference arm: a deliberately plain program).
 lookup protocol's Steps 2 and 3 composed from plaintext products, blind
 rotations of GLWE test polynomials, a key switch and RLWE traces) on the
 same ring, four segments, one line of its own; `--path multi_lut` the PBS
-with a LUT per ciphertext (four LUTs in one launch).
+with a LUT per ciphertext (four LUTs in one launch); `--path peaks` the
+integer issue rates of the GPU (operations per clock per SM for IADD3, LOP3,
+IMAD, IMAD.HI, IMAD.WIDE, an IMAD+IADD3 mix and the NTT butterfly).
 """
 
 from __future__ import annotations
@@ -146,6 +148,48 @@ def peaks():
         return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
     except OSError:
         return {}
+
+
+# ---------------------------------------------------------------------------- integer issue rates
+
+INT_OPS = {0: "IADD3", 1: "LOP3", 2: "IMAD", 3: "IMAD.HI", 4: "IMAD.WIDE", 5: "IMAD+IADD3", 6: "butterfly"}
+
+
+def measure_int_rates(torch, dev, iters: int = 16384) -> dict:
+    """32-bit integer operations retired per clock per SM for each class
+    (libintpeaks.so: eight independent inline-PTX chains per thread, 4 CTAs
+    of 512 threads per SM).  The rate uses the SM clock the kernels
+    themselves saw (clock64 over %globaltimer), so it does not depend on the
+    clock the run happened to get; `mhz` reports that clock."""
+    import ctypes
+    from paper_2609_16915_gb300 import build as B
+    L = ctypes.CDLL(B.build_peaks())
+    L.intpeak_launch.argtypes = [ctypes.c_int, ctypes.c_uint32, ctypes.c_uint32, ctypes.c_uint32, ctypes.c_void_p,
+                                 ctypes.c_void_p, ctypes.c_void_p]
+    L.intpeak_ops_per_iter.restype = ctypes.c_uint32
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    ctas, threads = 4 * sms, 512
+    sink = torch.zeros(1, dtype=torch.int32, device=dev)
+    stamps = torch.zeros(2 * ctas, dtype=torch.int64, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    out = {}
+    for op, name in INT_OPS.items():
+        # one untimed launch, then the timed one
+        st = L.intpeak_launch(op, ctas, threads, iters, sink.data_ptr(), stamps.data_ptr(), stream.cuda_stream)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        st = st or L.intpeak_launch(op, ctas, threads, iters, sink.data_ptr(), stamps.data_ptr(), stream.cuda_stream)
+        b.record(stream)
+        torch.cuda.synchronize(dev)
+        if st != 0:
+            raise RuntimeError(f"intpeak_launch({name}) failed: cudaError {st}")
+        ms = a.elapsed_time(b)
+        st = stamps.cpu().numpy().reshape(ctas, 2).astype(np.float64)
+        mhz = float(np.median(st[:, 0] / st[:, 1]) * 1e3)
+        ops = float(L.intpeak_ops_per_iter(op)) * iters * threads * ctas
+        out[name] = {"per_clk_per_sm": ops / (ms * 1e-3 * sms * mhz * 1e6), "mhz": mhz, "ms": ms}
+    out["sms"] = sms
+    return out
 
 
 # ---------------------------------------------------------------------------- clocks
@@ -401,18 +445,24 @@ def main():
     ap.add_argument("--batch", type=int, default=0, help="override the workload's batch")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-sample", type=int, default=0, help="oracle sample size (default: three per host core)")
-    ap.add_argument("--path", default="pbs", choices=["pbs", "lookup", "multi_lut"])
+    ap.add_argument("--path", default="pbs", choices=["pbs", "lookup", "multi_lut", "peaks"])
     args = ap.parse_args()
     p = W.CONFIGS[args.config]
     batch = args.batch or p.batch
     if args.impl == "reference":
         return run_reference(args, p, batch)
-    if args.path in ("lookup", "multi_lut"):
+    if args.path in ("lookup", "multi_lut", "peaks"):
         import torch
         import paper_2609_16915_gb300 as R
         R.load()
         dev = torch.device("cuda", 0)
         torch.cuda.set_device(dev)
+        if args.path == "peaks":
+            with ClockSampler(0) as clk:
+                rates = measure_int_rates(torch, dev)
+            print(json.dumps({"metric": "32-bit integer operations per clock per SM", "rates": rates,
+                              "clocks": clk.summary()}), flush=True)
+            return None
         if args.path == "lookup":
             return run_lookup(args, p, args.batch or 1024, torch, dev, R, ClockSampler)
         return run_multi_lut(args, p, batch, torch, dev, R, ClockSampler)
@@ -513,6 +563,10 @@ def main():
     alu_peak = sms * 128 * sm_max * 1e6 / 1e12   # T int32 ops/s: SMs x 128 lanes x max clock
     br_ops, ks_ops = int_ops_per_pbs(p)
     achieved = br_ops * batch / (br_ms / 1e3) / 1e12
+    # measured issue rate of the NTT butterfly's instruction mix (three
+    # multiplies, two adds) on this GPU, at the same maximum clock
+    rates = measure_int_rates(torch, dev)
+    mix_peak = rates["butterfly"]["per_clk_per_sm"] * sms * sm_max * 1e6 / 1e12
     pbs_roof = alu_peak * 1e12 / (br_ops + ks_ops)
     limbs = ks_tensor_limbs(p, batch)
     if limbs:
@@ -540,7 +594,10 @@ def main():
                      "unit": "Tops/s (int32)", "frac": achieved / alu_peak, "traffic": measured_traffic(p, batch),
                      "peak_basis": f"{sms} SMs x 128 int32 lanes x {sm_max:.0f} MHz (sm_max_mhz of MEASURED_PEAKS.json)",
                      "kernel_ms": br_ms, "keyswitch_ms": ks_ms, "keyswitch": ks_roof,
-                     "pbs_roof": pbs_roof, "pbs_frac_of_roof": value / world / pbs_roof},
+                     "pbs_roof": pbs_roof, "pbs_frac_of_roof": value / world / pbs_roof,
+                     "measured_mix_peak": mix_peak, "frac_of_measured_mix_peak": achieved / mix_peak,
+                     "int_rates_per_clk_per_sm": {k: round(v["per_clk_per_sm"], 2) for k, v in rates.items()
+                                                  if isinstance(v, dict)}},
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": batch * (p.n + 1) * 8 + lut.numel() * 8,
                 "d2h_bytes_per_step": batch * (p.n + 1) * 8},
         "gpu_launches": (3 if limbs else 2) * args.steps,

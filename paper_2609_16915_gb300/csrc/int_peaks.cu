@@ -138,6 +138,55 @@ __global__ void __launch_bounds__(512) bfly_peak_kernel(uint32_t iters, uint32_t
   }
 }
 
+// The butterfly three primes near 2^31 would need (products of three such
+// primes reach the 92-93 bits the larger parameter sets ask for): 4p no
+// longer fits 32 bits, so t and X are brought below p in every butterfly
+// before the adds: t = min(t, t - p), X = min(X, X - p), X' = X + t,
+// Y' = X - t + p, with the same Shoup product.  Counted as 9 integer
+// operations (three multiplies, six adds and minima).
+__global__ void __launch_bounds__(512) bfly31_peak_kernel(uint32_t iters, uint32_t seed, uint32_t *sink,
+                                                          unsigned long long *stamps) {
+  const uint32_t p = 2147352577u;  // 2^31 - 2^17 + 1
+  uint32_t X[kChains], Y[kChains];
+#pragma unroll
+  for (int j = 0; j < kChains; ++j) {
+    X[j] = (seed ^ (threadIdx.x * 2654435761u) ^ j) % (2 * p);
+    Y[j] = (seed * 7u + threadIdx.x + j * 977u) % (2 * p);
+  }
+  const uint32_t w = (seed % p) | 1u;
+  const uint32_t ws = static_cast<uint32_t>((static_cast<uint64_t>(w) << 32) / p);
+  __syncthreads();
+  const long long c0 = clock64();
+  const uint64_t g0 = globaltimer();
+  for (uint32_t i = 0; i < iters; ++i) {
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+#pragma unroll
+      for (int j = 0; j < kChains; ++j) {
+        uint32_t q, t;
+        asm volatile("mul.hi.u32 %0, %1, %2;" : "=r"(q) : "r"(Y[j]), "r"(ws));
+        asm volatile("{ .reg .u32 m; mul.lo.u32 m, %1, %2; mad.lo.u32 %0, %3, %4, m; }"
+                     : "=r"(t)
+                     : "r"(Y[j]), "r"(w), "r"(q), "r"(0u - p));
+        t = min(t, t - p);
+        const uint32_t x = min(X[j], X[j] - p);
+        X[j] = x + t;
+        Y[j] = x - t + p;
+      }
+  }
+  __syncthreads();
+  const long long c1 = clock64();
+  const uint64_t g1 = globaltimer();
+  uint32_t r = 0;
+#pragma unroll
+  for (int j = 0; j < kChains; ++j) r ^= X[j] ^ Y[j];
+  if (r == 0x9e3779b9u) sink[0] = r;
+  if (threadIdx.x == 0) {
+    stamps[2 * blockIdx.x] = static_cast<unsigned long long>(c1 - c0);
+    stamps[2 * blockIdx.x + 1] = g1 - g0;
+  }
+}
+
 // IMAD.WIDE: 64-bit chains acc = lo(acc) a + acc, so both halves of every
 // 32 x 32 -> 64 product are live.
 __global__ void __launch_bounds__(512) wide_peak_kernel(uint32_t iters, uint32_t seed, uint32_t *sink,
@@ -173,13 +222,15 @@ __global__ void __launch_bounds__(512) wide_peak_kernel(uint32_t iters, uint32_t
 
 // Integer operations one thread executes per loop iteration of kernel `op`
 // (0 IADD3, 1 LOP3, 2 IMAD, 3 IMAD.HI, 4 IMAD.WIDE, 5 IMAD+IADD3,
-// 6 butterfly: 5 integer operations);
+// 6 butterfly: 5 integer operations, 7 the butterfly of primes near 2^31:
+// 9 integer operations);
 // 0 for an unknown op.
 extern "C" uint32_t intpeak_ops_per_iter(int op) {
   switch (op) {
     case 0: case 1: case 2: case 3: case 4: return 4 * kChains;
     case 5: return 4 * kChains * 2;
     case 6: return 4 * kChains * 5;
+    case 7: return 4 * kChains * 9;
     default: return 0;
   }
 }
@@ -201,6 +252,7 @@ extern "C" int intpeak_launch(int op, uint32_t ctas, uint32_t threads, uint32_t 
     case 4: wide_peak_kernel<<<ctas, threads, 0, s>>>(iters, seed, sink, stamps); break;
     case 5: int_peak_kernel<5><<<ctas, threads, 0, s>>>(iters, seed, sink, stamps); break;
     case 6: bfly_peak_kernel<<<ctas, threads, 0, s>>>(iters, seed, sink, stamps); break;
+    case 7: bfly31_peak_kernel<<<ctas, threads, 0, s>>>(iters, seed, sink, stamps); break;
     default: return cudaErrorInvalidValue;
   }
   return static_cast<int>(cudaGetLastError());

@@ -376,7 +376,7 @@ def run_lookup(args, p, batch, torch, dev, R, clock_sampler):
         "gpu_launches": (4 * n_seg + 6) * args.steps,
         "clocks": clk.summary(),
     }
-    print(json.dumps(line), flush=True)
+    return line
 
 
 # ---------------------------------------------------------------------------- many-LUT path
@@ -432,7 +432,79 @@ def run_multi_lut(args, p, batch, torch, dev, R, clock_sampler):
         "gpu_launches": (3 if ks_tensor_limbs(p, batch) else 2) * args.steps,
         "clocks": clk.summary(),
     }
-    print(json.dumps(line), flush=True)
+    return line
+
+
+# ---------------------------------------------------------------------------- other workloads, same run
+
+class _Steps:
+    """argparse-like holder for the short runs of the other workloads."""
+
+    def __init__(self, steps, warmup):
+        self.steps, self.warmup = steps, warmup
+
+
+class _NoClock:
+    def __init__(self, *_):
+        pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *_):
+        pass
+
+    def summary(self):
+        return None
+
+
+def measure_other_config(name, torch, dev, R, steps, warmup, sms, sm_max, bfly_per_clk):
+    """PBS/s of another parameter set at its full batch (uniform-word keys and
+    ciphertexts resident, L2 flushed between steps), the blind rotation timed
+    alone, and its fractions of the two peaks."""
+    p = W.CONFIGS[name]
+    batch = p.batch
+
+    def d(a):
+        return torch.from_numpy(np.ascontiguousarray(a).view(np.int64)).to(dev)
+
+    bsk, ksk = W.uniform_keys(p)
+    ctx = R.Context(p, device=dev.index or 0, max_batch=batch)
+    ctx.upload_bsk(d(bsk))
+    ctx.upload_ksk(d(ksk))
+    del bsk, ksk
+    lwe = d(W.uniform_ciphertexts(p, batch, sub=1))
+    lut = d(W.lut_torus(p))
+    out = torch.empty((batch, p.n + 1), dtype=torch.int64, device=dev)
+    big = torch.empty((batch, p.kN + 1), dtype=torch.int64, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.int32, device=dev)
+    for _ in range(warmup):
+        ctx.pbs_batch(lwe, lut, out, stream)
+    ctx.sync_status(stream)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    for a, b in ev:
+        flush.zero_()
+        a.record(stream)
+        ctx.pbs_batch(lwe, lut, out, stream)
+        b.record(stream)
+    flush.zero_()
+    a1, b1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a1.record(stream)
+    ctx.blind_rotate_extract_batch(lwe, lut, big, stream)
+    b1.record(stream)
+    ctx.sync_status(stream)
+    ms = sum(a.elapsed_time(b) for a, b in ev) / steps
+    br_ms = a1.elapsed_time(b1)
+    br_ops, _ = int_ops_per_pbs(p)
+    achieved = br_ops * batch / (br_ms / 1e3) / 1e12
+    ctx.close()
+    del lwe, out, big, flush
+    torch.cuda.empty_cache()
+    return {"workload": describe(p, batch), "value": batch / (ms / 1e3), "unit": UNIT, "ms_per_step": ms,
+            "steps": steps, "warmup": warmup, "blind_rotation_ms": br_ms, "achieved_tops": achieved,
+            "frac": achieved / (sms * 128 * sm_max * 1e6 / 1e12),
+            "frac_of_butterfly_rate_peak": achieved / (bfly_per_clk * 8 * sms * sm_max * 1e6 / 1e12)}
 
 
 # ---------------------------------------------------------------------------- GPU arm
@@ -446,6 +518,8 @@ def main():
     ap.add_argument("--config", default="standard", choices=sorted(W.CONFIGS))
     ap.add_argument("--batch", type=int, default=0, help="override the workload's batch")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-other", action="store_true",
+                    help="skip the short runs of the other parameter sets and paths that follow the headline")
     ap.add_argument("--cpu-sample", type=int, default=0, help="oracle sample size (default: three per host core)")
     ap.add_argument("--path", default="pbs", choices=["pbs", "lookup", "multi_lut", "peaks"])
     args = ap.parse_args()
@@ -466,8 +540,11 @@ def main():
                               "clocks": clk.summary()}), flush=True)
             return None
         if args.path == "lookup":
-            return run_lookup(args, p, args.batch or 1024, torch, dev, R, ClockSampler)
-        return run_multi_lut(args, p, batch, torch, dev, R, ClockSampler)
+            line = run_lookup(args, p, args.batch or 1024, torch, dev, R, ClockSampler)
+        else:
+            line = run_multi_lut(args, p, batch, torch, dev, R, ClockSampler)
+        print(json.dumps(line), flush=True)
+        return None
 
     import torch
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -610,6 +687,21 @@ def main():
         "clocks": clk.summary(),
         "wall_s_timed": wall,
     }
+    if world == 1 and not args.no_other and args.config == "standard" and not args.batch:
+        # the other rows, measured in the same run after the headline's timed
+        # region (short runs: their own warm-up and steps, L2 flushed between
+        # steps); uniform-word keys as above
+        other = {}
+        for name, st, wu in (("gpt2_mlp", 3, 2), ("llama_silu", 2, 1)):
+            other[name] = measure_other_config(name, torch, dev, R, st, wu, sms, sm_max, bfly_per_clk)
+        ml = run_multi_lut(_Steps(2, 1), p, batch, torch, dev, R, _NoClock)
+        other["multi_lut"] = {k: ml[k] for k in ("metric", "value", "unit", "ms_per_step", "steps")}
+        other["multi_lut"]["workload"] = ml["config"]["workload"]
+        lk = run_lookup(_Steps(2, 1), p, 1024, torch, dev, R, _NoClock)
+        other["lookup"] = {k: lk[k] for k in ("metric", "value", "unit", "ms_per_step", "steps")}
+        other["lookup"]["workload"] = lk["config"]["workload"]
+        other["lookup"]["blind_rotation_frac"] = lk["roofline"]["frac"]
+        line["other_workloads"] = other
     if not args.no_cpu_baseline:
         import oracle as O
         O.build()

@@ -72,7 +72,8 @@ typedef enum {
   ROSETTA_ERR_KEYS_MISSING = -3,       /* BSK or KSK not uploaded */
   ROSETTA_ERR_CUDA = -4,               /* a CUDA runtime call or launch failed */
   ROSETTA_ERR_OOM = -5,                /* device allocation failed */
-  ROSETTA_ERR_TIMEOUT = -6             /* a bounded device-side wait expired */
+  ROSETTA_ERR_TIMEOUT = -6,            /* a bounded device-side wait expired */
+  ROSETTA_ERR_BOUNDS = -7              /* a device-side bounds check of a ROSETTA_DEBUG build failed */
 } rosetta_status;
 
 typedef struct rosetta_ctx rosetta_ctx; /* opaque, library-owned */
@@ -280,11 +281,25 @@ int rosetta_pbs_batch_noalloc(rosetta_ctx *ctx, const uint64_t *lwe_in, uint32_t
  * INVALID_ARG, CUDA. */
 int rosetta_selftest_wait_timeout(rosetta_ctx *ctx, uint32_t limit_us, void *stream);
 
+/* Self-test of the bounds checks of a library compiled with -DROSETTA_DEBUG
+ * (no counterpart in the paper; that build stands in for a memory checker,
+ * which this GPU pool does not offer).  The debug kernels compare the key
+ * block each CMux step reads with the size of the transformed key and each
+ * cluster's ciphertext index with the batch; a failed check skips the access
+ * and raises the context's error flag, so rosetta_sync_status returns
+ * ROSETTA_ERR_BOUNDS once and the context stays usable (nothing traps).
+ * This call blind-rotates one ciphertext, with only its last mask word
+ * nonzero, with the key declared one step shorter than it is, so the last
+ * step's check fails.  Needs the BSK.  Regular build: UNSUPPORTED_PARAMS.
+ * Errors: INVALID_ARG, KEYS_MISSING, CUDA, OOM. */
+int rosetta_selftest_bounds(rosetta_ctx *ctx, void *stream);
+
 /* Wait for all work on `stream` and report any deferred execution error
  * (CUDA; TIMEOUT when a bounded wait of the tensor-core key switch gave up;
  * INVALID_ARG for an out-of-range LUT index seen by
- * rosetta_pbs_batch_multi_lut; the flag is cleared once reported).  Returns
- * OK when the stream finished cleanly. */
+ * rosetta_pbs_batch_multi_lut; BOUNDS when a check of a ROSETTA_DEBUG build
+ * failed; the flag is cleared once reported).  Returns OK when the stream
+ * finished cleanly. */
 int rosetta_sync_status(rosetta_ctx *ctx, void *stream);
 
 /* Free everything the context owns.  Waits for the context's device work.

@@ -15,16 +15,19 @@ import os
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "librosetta.so")
+# the same library compiled with -DROSETTA_DEBUG (device-side bounds checks)
+DEBUG_LIB_PATH = os.path.join(_HERE, "librosetta_debug.so")
 
 ROSETTA_OK = 0
 STATUS = {0: "ok", -1: "invalid argument", -2: "unsupported parameters", -3: "keys not uploaded",
-          -4: "CUDA error", -5: "out of device memory", -6: "device wait timed out"}
+          -4: "CUDA error", -5: "out of device memory", -6: "device wait timed out",
+          -7: "device-side bounds check failed (debug build)"}
 
 EXPORTS = ("rosetta_params_init", "rosetta_upload_bsk", "rosetta_upload_ksk", "rosetta_pbs_batch",
            "rosetta_blind_rotate_extract_batch", "rosetta_keyswitch_batch", "rosetta_pbs_batch_multi_lut",
            "rosetta_blind_rotate_glwe_batch", "rosetta_upload_trace_keys", "rosetta_trace_batch",
            "rosetta_plaintext_mul_batch", "rosetta_upload_lookup_table", "rosetta_segmented_lookup_batch",
-           "rosetta_selftest_wait_timeout",
+           "rosetta_selftest_wait_timeout", "rosetta_selftest_bounds",
            "rosetta_pbs_batch_noalloc",
            "rosetta_sync_status", "rosetta_destroy", "rosetta_status_string")
 
@@ -68,6 +71,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     L.rosetta_upload_lookup_table.argtypes = [vp, u32, u64p, u64p, u64p, u64p, vp]
     L.rosetta_segmented_lookup_batch.argtypes = [vp, u64p, u64p, u32, u64p, vp]
     L.rosetta_selftest_wait_timeout.argtypes = [vp, u32, vp]
+    L.rosetta_selftest_bounds.argtypes = [vp, vp]
     L.rosetta_sync_status.argtypes = [vp, vp]
     L.rosetta_destroy.argtypes = [vp]
     L.rosetta_destroy.restype = None
@@ -234,6 +238,11 @@ class Context:
         _check("rosetta_selftest_wait_timeout",
                load().rosetta_selftest_wait_timeout(self._h, limit_us, _stream(stream)))
 
+    def rosetta_selftest_bounds(self, stream=None):
+        """Make one bounds check of a ROSETTA_DEBUG build fail (reported by
+        sync_status as BOUNDS); the regular build returns UNSUPPORTED_PARAMS."""
+        _check("rosetta_selftest_bounds", load().rosetta_selftest_bounds(self._h, _stream(stream)))
+
     def rosetta_pbs_batch_noalloc(self, lwe_in, lut, lwe_out, stream=None):
         """rosetta_pbs_batch without any device allocation in the call (fixed
         in-library scratch; device buffers only, bounded batch)."""
@@ -259,4 +268,5 @@ class Context:
     upload_lookup_table = rosetta_upload_lookup_table
     segmented_lookup_batch = rosetta_segmented_lookup_batch
     selftest_wait_timeout = rosetta_selftest_wait_timeout
+    selftest_bounds = rosetta_selftest_bounds
     sync_status = rosetta_sync_status

@@ -15,6 +15,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 ROOT = os.path.dirname(HERE)
 LIB = os.path.join(HERE, "librosetta.so")
+DEBUG_LIB = os.path.join(HERE, "librosetta_debug.so")
 BUILD_DIR = os.path.join(ROOT, "_build")
 SOURCES = ["tables.cu", "bsk_transform.cu", "blind_rotate.cu", "keyswitch.cu", "keyswitch_tc.cu", "rosetta_api.cu",
            "pbs_noalloc.cu", "trace.cu"]
@@ -35,10 +36,10 @@ def _flags(verbose: bool):
     return f
 
 
-def _stale(objs) -> bool:
-    if not os.path.exists(LIB):
+def _stale(objs, lib) -> bool:
+    if not os.path.exists(lib):
         return True
-    t = os.path.getmtime(LIB)
+    t = os.path.getmtime(lib)
     deps = [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f != PEAKS_SRC] + [os.path.join(ROOT, "include", "rosetta.h"),
                                                                                  __file__]
     return any(os.path.getmtime(d) > t for d in deps)
@@ -64,16 +65,22 @@ def build_peaks(force: bool = False) -> str:
     return PEAKS_LIB
 
 
-def build(force: bool = False, verbose: bool = False) -> str:
-    os.makedirs(BUILD_DIR, exist_ok=True)
-    objs = [os.path.join(BUILD_DIR, s.replace(".cu", ".o")) for s in SOURCES]
-    if not force and not _stale(objs):
-        return LIB
+def build(force: bool = False, verbose: bool = False, debug: bool = False) -> str:
+    """Build librosetta.so, or with debug=True librosetta_debug.so: the same
+    sources compiled with -DROSETTA_DEBUG (device-side bounds checks that
+    report ROSETTA_ERR_BOUNDS instead of reading outside a buffer)."""
+    lib = DEBUG_LIB if debug else LIB
+    bdir = os.path.join(BUILD_DIR, "debug") if debug else BUILD_DIR
+    os.makedirs(bdir, exist_ok=True)
+    objs = [os.path.join(bdir, s.replace(".cu", ".o")) for s in SOURCES]
+    if not force and not _stale(objs, lib):
+        return lib
     cc = nvcc()
+    extra = ["-DROSETTA_DEBUG"] if debug else []
 
     def compile_one(src_obj):
         src, obj = src_obj
-        cmd = [cc, "-c", os.path.join(CSRC, src), "-o", obj] + _flags(verbose)
+        cmd = [cc, "-c", os.path.join(CSRC, src), "-o", obj] + _flags(verbose) + extra
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
             raise RuntimeError(f"nvcc failed for {src}:\n{r.stdout}\n{r.stderr}")
@@ -84,15 +91,15 @@ def build(force: bool = False, verbose: bool = False) -> str:
     if verbose:
         for s, log in zip(SOURCES, logs):
             print(f"--- {s}\n{log}")
-    tmp = LIB + f".tmp{os.getpid()}"
+    tmp = lib + f".tmp{os.getpid()}"
     cmd = [cc, "-shared", "-o", tmp] + objs + ARCH + ["-lcudart"]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
-    os.replace(tmp, LIB)
-    return LIB
+    os.replace(tmp, lib)
+    return lib
 
 
 if __name__ == "__main__":
     import sys
-    print(build(force=True, verbose="-v" in sys.argv))
+    print(build(force=True, verbose="-v" in sys.argv, debug="--debug" in sys.argv))

@@ -34,6 +34,7 @@
 
 #include <type_traits>
 
+#include "check.cuh"
 #include "dsmem.cuh"
 #include "internal.h"
 #include "ntt.cuh"
@@ -80,6 +81,7 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
   const uint32_t rank = cluster.block_rank();
   const uint32_t ct = blockIdx.x / 4;
   const uint32_t tau = threadIdx.x;
+  if (!dbg_ok(ct < a.batch, a.err_flag)) return;  // the whole cluster shares ct
 
   extern __shared__ __align__(16) unsigned char smem[];
   uint2 *tw = reinterpret_cast<uint2 *>(smem);                   // [N]
@@ -236,7 +238,10 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
 
     // ---- phase 2: transforms and pointwise products for prime `rank` ----
     uint32_t oh[2][E];
-    const uint32_t *gbase = a.bsk + (static_cast<size_t>(i) * kPrimes + rank) * (static_cast<size_t>(L2) * 2 * N);
+    const size_t kblk = static_cast<size_t>(L2) * 2 * N;  // words of one step's key block per prime
+    const uint32_t *gbase = a.bsk + (static_cast<size_t>(i) * kPrimes + rank) * kblk;
+    const bool key_ok = dbg_ok(a.bsk_words == 0 || (static_cast<size_t>(i) * kPrimes + rank + 1) * kblk <= a.bsk_words,
+                               a.err_flag);
 #pragma unroll 1
     for (uint32_t r0 = 0; r0 < L2; r0 += 2) {
       // first-pass slot q of thread tau is coefficient tau + q N/E, owned by
@@ -278,7 +283,8 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
         uint32_t ga[E], gb[E];
 #pragma unroll
         for (int k = 0; k < E / 4; ++k) {
-          const uint4 va = __ldg(g + (c * N) / 4 + k), vb = __ldg(g + ((2 + c) * N) / 4 + k);
+          const uint4 va = key_ok ? __ldg(g + (c * N) / 4 + k) : make_uint4(0u, 0u, 0u, 0u);
+          const uint4 vb = key_ok ? __ldg(g + ((2 + c) * N) / 4 + k) : make_uint4(0u, 0u, 0u, 0u);
           ga[4 * k] = va.x; ga[4 * k + 1] = va.y; ga[4 * k + 2] = va.z; ga[4 * k + 3] = va.w;
           gb[4 * k] = vb.x; gb[4 * k + 1] = vb.y; gb[4 * k + 2] = vb.z; gb[4 * k + 3] = vb.w;
         }

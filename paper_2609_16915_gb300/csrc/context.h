@@ -16,6 +16,7 @@ struct rosetta_ctx {
   rosetta::CrtConsts cc{};
   uint2 *d_tw = nullptr;          // [kPrimes][N]
   uint32_t *d_bsk = nullptr;      // transform domain
+  size_t bsk_words = 0;           // its size in 32-bit words
   uint64_t *d_ksk = nullptr;      // raw [kN][l_ks][n+1]
   uint64_t *d_corr = nullptr;     // [n+1]
   uint16_t *d_ks_b = nullptr;     // key limb tiles for the tensor-core key switch (null: not exact)

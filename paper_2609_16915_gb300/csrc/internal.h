@@ -38,6 +38,7 @@ struct BrArgs {
   const uint64_t *glwe_in;  // [batch][2][N] GLWE test polynomials, or null
   uint32_t *err_flag;       // set to 1 when a LUT index is out of range
   const uint32_t *bsk;      // transform domain [n][prime][2l][2][N]
+  size_t bsk_words;         // words of bsk (checked by ROSETTA_DEBUG builds; 0: unchecked)
   const uint2 *tw;          // [prime][N] (W, Shoup companion)
   uint32_t n, level, base_log, msg_bits, batch, num_luts;
   CrtConsts cc;

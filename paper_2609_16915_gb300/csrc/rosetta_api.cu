@@ -158,6 +158,7 @@ BrArgs br_args(const rosetta_ctx *c, const uint64_t *in, uint32_t batch, const u
   a.lut = lut;
   a.lwe_big_out = big;
   a.bsk = c->d_bsk;
+  a.bsk_words = c->bsk_words;
   a.tw = c->d_tw;
   a.n = c->prm.lwe_dim;
   a.level = c->prm.pbs_level;
@@ -267,6 +268,7 @@ const char *rosetta_status_string(int status) {
     case ROSETTA_ERR_CUDA: return "CUDA error";
     case ROSETTA_ERR_OOM: return "out of device memory";
     case ROSETTA_ERR_TIMEOUT: return "device wait timed out";
+    case ROSETTA_ERR_BOUNDS: return "device-side bounds check failed (debug build)";
     default: return "unknown status";
   }
 }
@@ -355,6 +357,7 @@ int rosetta_upload_bsk(rosetta_ctx *c, const uint64_t *bsk, size_t n_words, int 
     e = cudaStreamSynchronize(s);  // caller may free the host buffer on return
     if (e != cudaSuccess) return cuda_fail(e);
   }
+  c->bsk_words = want * kPrimes;
   c->have_bsk = true;
   return ROSETTA_OK;
 }
@@ -717,8 +720,42 @@ int rosetta_sync_status(rosetta_ctx *c, void *stream) {
   e = cudaMemcpy(&flag, c->d_err, sizeof(flag), cudaMemcpyDeviceToHost);
   if (e == cudaSuccess && flag) e = cudaMemset(c->d_err, 0, sizeof(flag));
   if (e != cudaSuccess) return cuda_fail(e);
-  // 1: a LUT index out of range; 2: a bounded device-side wait gave up
-  return flag == 2 ? ROSETTA_ERR_TIMEOUT : (flag ? ROSETTA_ERR_INVALID_ARG : ROSETTA_OK);
+  // 1: a LUT index out of range; 2: a bounded device-side wait gave up;
+  // 3: a bounds check of a ROSETTA_DEBUG build failed (the access was skipped)
+  if (flag == 2) return ROSETTA_ERR_TIMEOUT;
+  if (flag == 3) return ROSETTA_ERR_BOUNDS;
+  return flag ? ROSETTA_ERR_INVALID_ARG : ROSETTA_OK;
+}
+
+int rosetta_selftest_bounds(rosetta_ctx *c, void *stream) {
+  if (!c) return ROSETTA_ERR_INVALID_ARG;
+#ifndef ROSETTA_DEBUG
+  (void)stream;
+  return ROSETTA_ERR_UNSUPPORTED_PARAMS;  // the checks exist only in a ROSETTA_DEBUG build
+#else
+  if (!c->have_bsk) return ROSETTA_ERR_KEYS_MISSING;
+  if (cudaSetDevice(c->device) != cudaSuccess) return ROSETTA_ERR_CUDA;
+  const cudaStream_t s = as_stream(stream);
+  // One ciphertext whose only nonzero mask word is the last (a~ = N, so only
+  // the last CMux step runs), blind-rotated with the transformed key declared
+  // one step's block shorter than it is: that step's key block fails its
+  // check, the kernel skips the loads (it reads nothing past what it is
+  // told exists) and raises the flag.
+  int r = ensure_stage(c, 1, s);
+  if (r == ROSETTA_OK) r = ensure_big(c, 1, s);
+  if (r != ROSETTA_OK) return r;
+  const uint64_t word = 1ull << 63;
+  cudaError_t e = cudaMemsetAsync(c->d_in, 0, lwe_words(c) * sizeof(uint64_t), s);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(c->d_in + c->prm.lwe_dim - 1, &word, sizeof(word), cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(c->d_lut, 0, sizeof(uint64_t) << c->prm.msg_bits, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);  // `word` lives on this stack frame
+  if (e != cudaSuccess) return cuda_fail(e);
+  BrArgs a = br_args(c, c->d_in, 1, c->d_lut, c->d_big);
+  const size_t step = c->bsk_words / c->prm.lwe_dim;
+  a.bsk_words = c->bsk_words - step;
+  e = launch_blind_rotate(a, c->logN, c->dig16, s);
+  return e == cudaSuccess ? ROSETTA_OK : cuda_fail(e);
+#endif
 }
 
 void rosetta_destroy(rosetta_ctx *c) {

@@ -112,3 +112,15 @@ def test_binding_argument_counts_match_the_header(lib):
     assert set(arity) == set(declared_functions())
     for name, n in arity.items():
         assert len(getattr(lib, name).argtypes) == n, name
+
+
+def test_debug_build_compiles_and_exports_the_same_symbols(lib):
+    """The ROSETTA_DEBUG library (device-side bounds checks) builds from the
+    same sources and has the same boundary."""
+    from paper_2609_16915_gb300 import build
+    path = build.build(debug=True)
+    dbg = ctypes.CDLL(path)
+    for name in declared_functions():
+        assert hasattr(dbg, name), name
+    dbg.rosetta_status_string.restype = ctypes.c_char_p
+    assert dbg.rosetta_status_string(-7) == b"device-side bounds check failed (debug build)"

@@ -103,10 +103,21 @@ typedef struct {
  * beta > 16.  Errors: INVALID_ARG (NULL), UNSUPPORTED_PARAMS, CUDA, OOM. */
 int rosetta_params_init(rosetta_ctx **out, const rosetta_params *p, int cuda_device);
 
+/* Number of NTT primes the context's blind rotation computes the external
+ * product over: 4 (primes just below 2^28, one CTA per prime in a cluster of
+ * four) or 3 (primes just below 2^31, a cluster of three).  The context takes
+ * three where (k+1) l N 2^(beta-1) 2^63 <= 0.45 x 2^92.999 (the three primes'
+ * product), a three-prime kernel exists (N = 4096, beta <= 16, l <= 2) and two
+ * of its CTAs fit one SM's shared memory (on a 228 KB SM: n <= 1535 at l = 2,
+ * n <= 4607 at l = 1); e.g. N = 4096, l = 2, beta = 15.  Either way the outputs are the same words: the
+ * product is exact.  Fixed at rosetta_params_init.  Returns 3 or 4, or
+ * INVALID_ARG for a NULL context. */
+int rosetta_ntt_primes(const rosetta_ctx *ctx);
+
 /* Upload the raw bootstrapping key (layout above, n_words =
  * n*(k+1)*l*(k+1)*N) and convert it on the device to the transform domain
  * used by the external product (per-prime negacyclic NTT of the centred
- * words).  The source may be host or device memory (src_is_device selects);
+ * words, over the context's rosetta_ntt_primes primes).  The source may be host or device memory (src_is_device selects);
  * the caller keeps ownership and may free it after the call returns.  The
  * conversion is stream-ordered on `stream`.  Errors: INVALID_ARG, CUDA, OOM. */
 int rosetta_upload_bsk(rosetta_ctx *ctx, const uint64_t *bsk, size_t n_words,

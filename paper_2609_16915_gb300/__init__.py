@@ -28,7 +28,7 @@ EXPORTS = ("rosetta_params_init", "rosetta_upload_bsk", "rosetta_upload_ksk", "r
            "rosetta_blind_rotate_glwe_batch", "rosetta_upload_trace_keys", "rosetta_trace_batch",
            "rosetta_plaintext_mul_batch", "rosetta_upload_lookup_table", "rosetta_segmented_lookup_batch",
            "rosetta_selftest_wait_timeout", "rosetta_selftest_bounds",
-           "rosetta_pbs_batch_noalloc",
+           "rosetta_pbs_batch_noalloc", "rosetta_ntt_primes",
            "rosetta_sync_status", "rosetta_destroy", "rosetta_status_string")
 
 
@@ -72,6 +72,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     L.rosetta_segmented_lookup_batch.argtypes = [vp, u64p, u64p, u32, u64p, vp]
     L.rosetta_selftest_wait_timeout.argtypes = [vp, u32, vp]
     L.rosetta_selftest_bounds.argtypes = [vp, vp]
+    L.rosetta_ntt_primes.argtypes = [vp]
     L.rosetta_sync_status.argtypes = [vp, vp]
     L.rosetta_destroy.argtypes = [vp]
     L.rosetta_destroy.restype = None
@@ -251,6 +252,13 @@ class Context:
                                                                              _ptr(lwe_out), _stream(stream)))
         return lwe_out
 
+    def rosetta_ntt_primes(self):
+        """Primes of the blind rotation's exact external product: 3 or 4."""
+        r = load().rosetta_ntt_primes(self._h)
+        if r < 0:
+            raise RosettaError("rosetta_ntt_primes", r)
+        return r
+
     def rosetta_sync_status(self, stream=None):
         _check("rosetta_sync_status", load().rosetta_sync_status(self._h, _stream(stream)))
 
@@ -269,4 +277,5 @@ class Context:
     segmented_lookup_batch = rosetta_segmented_lookup_batch
     selftest_wait_timeout = rosetta_selftest_wait_timeout
     selftest_bounds = rosetta_selftest_bounds
+    ntt_primes = rosetta_ntt_primes
     sync_status = rosetta_sync_status

@@ -17,8 +17,8 @@ ROOT = os.path.dirname(HERE)
 LIB = os.path.join(HERE, "librosetta.so")
 DEBUG_LIB = os.path.join(HERE, "librosetta_debug.so")
 BUILD_DIR = os.path.join(ROOT, "_build")
-SOURCES = ["tables.cu", "bsk_transform.cu", "blind_rotate.cu", "keyswitch.cu", "keyswitch_tc.cu", "rosetta_api.cu",
-           "pbs_noalloc.cu", "trace.cu"]
+SOURCES = ["tables.cu", "bsk_transform.cu", "blind_rotate.cu", "blind_rotate3.cu", "keyswitch.cu", "keyswitch_tc.cu",
+           "rosetta_api.cu", "pbs_noalloc.cu", "trace.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

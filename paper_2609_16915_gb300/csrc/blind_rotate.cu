@@ -427,6 +427,8 @@ static cudaError_t launch_br_lev(const BrArgs &a, cudaStream_t s) {
 }
 
 cudaError_t launch_blind_rotate(const BrArgs &a, uint32_t logN, bool dig16, cudaStream_t s) {
+  if (a.primes == kPrimes31) return launch_blind_rotate3(a, logN, s);
+  if (a.primes != kPrimes) return cudaErrorInvalidValue;
 #define ROSETTA_BR_CASE(L)                                                        \
   case L:                                                                         \
     return dig16 ? launch_br_lev<L, true>(a, s) : launch_br_lev<L, false>(a, s);

@@ -15,7 +15,12 @@ struct rosetta_ctx {
   bool dig16 = false;
   rosetta::CrtConsts cc{};
   uint2 *d_tw = nullptr;          // [kPrimes][N]
-  uint32_t *d_bsk = nullptr;      // transform domain
+  // the blind rotation's prime set: kPrimes (d_tw, cc) or, where the
+  // external-product bound allows, the three 31-bit primes (d_tw31, cc31)
+  uint32_t br_primes = rosetta::kPrimes;
+  uint2 *d_tw31 = nullptr;        // [kPrimes31][N], or null
+  rosetta::CrtConsts cc31{};
+  uint32_t *d_bsk = nullptr;      // transform domain over br_primes primes
   size_t bsk_words = 0;           // its size in 32-bit words
   uint64_t *d_ksk = nullptr;      // raw [kN][l_ks][n+1]
   uint64_t *d_corr = nullptr;     // [n+1]
@@ -50,3 +55,14 @@ struct rosetta_ctx {
   uint64_t *d_lk_I = nullptr;     // interval-index LWEs [batch][n+1]
   size_t lk_I_cap = 0;
 };
+
+// The key, twiddle and CRT fields of a blind rotation over the context's
+// bootstrapping key.
+inline void br_key_args(const rosetta_ctx *c, rosetta::BrArgs *a) {
+  const bool three = c->br_primes == rosetta::kPrimes31;
+  a->bsk = c->d_bsk;
+  a->bsk_words = c->bsk_words;
+  a->primes = c->br_primes;
+  a->tw = three ? c->d_tw31 : c->d_tw;
+  a->cc = three ? c->cc31 : c->cc;
+}

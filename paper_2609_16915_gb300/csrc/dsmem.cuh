@@ -29,6 +29,12 @@ __device__ __forceinline__ int32_t dsmem_ld_s32(uint32_t a) {
   return v;
 }
 
+__device__ __forceinline__ uint32_t dsmem_ld_u32(uint32_t a) {
+  uint32_t v;
+  asm volatile("ld.shared::cluster.u32 %0, [%1];" : "=r"(v) : "r"(a) : "memory");
+  return v;
+}
+
 __device__ __forceinline__ int32_t dsmem_ld_s16(uint32_t a) {
   int32_t v;
   asm volatile("ld.shared::cluster.s16 %0, [%1];" : "=r"(v) : "r"(a) : "memory");
@@ -53,6 +59,10 @@ __device__ __forceinline__ uint2 dsmem_ld_v2_u32(uint32_t a) {
 __device__ __forceinline__ void dsmem_st_v4_u32(uint32_t a, uint4 v) {
   asm volatile("st.shared::cluster.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(a), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
                : "memory");
+}
+
+__device__ __forceinline__ void dsmem_st_v2_u32(uint32_t a, uint2 v) {
+  asm volatile("st.shared::cluster.v2.u32 [%0], {%1, %2};" ::"r"(a), "r"(v.x), "r"(v.y) : "memory");
 }
 
 __device__ __forceinline__ void dsmem_st_u32(uint32_t a, uint32_t v) {

@@ -14,6 +14,14 @@ namespace rosetta {
 constexpr int kPrimes = 4;
 constexpr uint32_t kPrimeList[kPrimes] = {268369921u, 268271617u, 268238849u, 268189697u};
 
+// Three NTT primes p = c * 2^14 + 1 in (2^31 - 2^19, 2^31), product
+// M > 2^92.999: the blind rotation's prime set for the parameter sets whose
+// external-product bound stays below 0.45 M (N = 4096 with (k+1) l 2^beta up
+// to 2^17, e.g. l = 2, beta = 15).  No lazy headroom (4p > 2^32): residues are
+// kept in [0, 2p).
+constexpr int kPrimes31 = 3;
+constexpr uint32_t kPrime31List[kPrimes31] = {2147352577u, 2147205121u, 2147074049u};
+
 struct PrimeConsts {
   uint32_t p;
   uint32_t p_inv;     // p^{-1} mod 2^32 (Montgomery reduction)
@@ -41,6 +49,7 @@ struct BrArgs {
   size_t bsk_words;         // words of bsk (checked by ROSETTA_DEBUG builds; 0: unchecked)
   const uint2 *tw;          // [prime][N] (W, Shoup companion)
   uint32_t n, level, base_log, msg_bits, batch, num_luts;
+  uint32_t primes;          // kPrimes (bsk, tw, cc over the 28-bit set) or kPrimes31
   CrtConsts cc;
 };
 
@@ -72,18 +81,26 @@ struct TraceArgs {
   CrtConsts cc;
 };
 
-// host-side tables (tables.cu)
-bool build_tables(uint32_t logN, uint2 *tw_host /*[kPrimes][N]*/, CrtConsts *cc);
+// host-side tables (tables.cu): twiddles and CRT constants of the 28-bit set
+// (primes = kPrimes) or of the 31-bit set (primes = kPrimes31)
+bool build_tables(uint32_t logN, uint32_t primes, uint2 *tw_host /*[primes][N]*/, CrtConsts *cc);
 
 // launchers; return cudaSuccess or the launch error
 size_t br_smem_bytes(uint32_t logN, uint32_t level, uint32_t n, bool dig16);
+// a.primes selects the kernel: the four-prime one or the three-prime one
 cudaError_t launch_blind_rotate(const BrArgs &a, uint32_t logN, bool dig16, cudaStream_t s);
+// three-prime kernel (blind_rotate3.cu): 16-bit digits, compiled ring sizes and levels only
+bool br3_supported(uint32_t logN, uint32_t level, bool dig16);
+size_t br3_smem_bytes(uint32_t logN, uint32_t level, uint32_t n);
+cudaError_t launch_blind_rotate3(const BrArgs &a, uint32_t logN, cudaStream_t s);
 cudaError_t launch_bsk_transform(const uint64_t *raw, uint32_t *out, const uint2 *tw, const CrtConsts &cc,
-                                 uint32_t logN, uint32_t n, uint32_t level, cudaStream_t s);
+                                 uint32_t logN, uint32_t n, uint32_t level, uint32_t primes, cudaStream_t s);
 cudaError_t launch_keyswitch(const KsArgs &a, cudaStream_t s);
 // transform `count` raw keys [count][rows][2][N] to [count][prime][rows][2][N]
+// over the 28-bit set (primes = kPrimes) or the 31-bit set (kPrimes31)
 cudaError_t launch_key_transform(const uint64_t *raw, uint32_t *out, const uint2 *tw, const CrtConsts &cc,
-                                 uint32_t logN, uint32_t count, uint32_t rows, cudaStream_t s);
+                                 uint32_t logN, uint32_t count, uint32_t rows, cudaStream_t s,
+                                 uint32_t primes = kPrimes);
 size_t trace_smem_bytes(uint32_t logN, uint32_t level);
 cudaError_t launch_trace(const TraceArgs &a, uint32_t logN, cudaStream_t s);
 cudaError_t launch_plaintext_mul(const TraceArgs &a, uint32_t logN, cudaStream_t s);

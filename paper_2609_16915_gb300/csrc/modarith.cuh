@@ -1,5 +1,6 @@
-// Word-level modular arithmetic for the NTT primes (p < 2^28, so 16p < 2^32
-// and lazily reduced residues up to 8p still fit a 32-bit register).
+// Word-level modular arithmetic for the NTT primes: the 28-bit set (16p <
+// 2^32, so lazily reduced residues up to 8p still fit a 32-bit register) and
+// the 31-bit set (2p < 2^32: residues below 2p).
 //
 // Residues are kept "lazy": a value congruent to the residue but possibly a
 // few multiples of p above it.  Every function states the range it accepts
@@ -33,6 +34,14 @@ __device__ __forceinline__ uint32_t redc(uint64_t T, uint32_t p, uint32_t p_inv)
 // bound every accepted parameter set meets), so the estimate stays within
 // 0.29 of that integer and rounds to it.
 __device__ __forceinline__ uint32_t crt_quotient(uint32_t ysum) { return (ysum + (1u << 25)) >> 26; }
+
+// The same for the three primes in (2^31 - 2^19, 2^31), from ysum = sum_q
+// (y_q >> 3) with every y_q < 2 p_q < 2^32 (the sum stays below 2^31).
+// y / 2^31 undershoots y / p by less than 2 (2^31 - p) / 2^31 < 2^-11 per
+// prime (the shift adds under 2^-28); the three together by less than 2^-9.
+// Only parameter sets whose exact integer value X obeys |X| <= 0.45 M take
+// this prime set, so the estimate stays within 0.46 of the integer.
+__device__ __forceinline__ uint32_t crt_quotient31(uint32_t ysum) { return (ysum + (1u << 27)) >> 28; }
 
 // x in [0, 2b) -> [0, b) for a bound b: one subtraction when x >= b.
 __device__ __forceinline__ uint32_t cond_sub(uint32_t x, uint32_t b) {

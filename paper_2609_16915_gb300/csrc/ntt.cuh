@@ -18,8 +18,10 @@
 // inverse pass needs, so a pointwise product between the two transforms
 // needs no exchange.
 //
-// Lazy ranges: forward input < 2p, output < 16p; inverse input < 4p, output
-// < 8p.  See the butterflies for the per-stage invariants.
+// Lazy ranges (primes below 2^28): forward input < 2p, output < 16p; inverse
+// input < 4p, output < 8p.  See the butterflies for the per-stage invariants.
+// With P31 (primes between 2^30 and 2^31, where 4p > 2^32 leaves no room for
+// lazy growth) every input and output lies in [0, 2p).
 #pragma once
 #include <stdint.h>
 
@@ -79,6 +81,24 @@ __device__ __forceinline__ void ct_bfly(uint32_t &X, uint32_t &Y, uint2 w, uint3
   X = X + t;
 }
 
+// Butterflies for primes 2^30 < p < 2^31, every value in [0, 2p).  Forward:
+// X' = x + t, Y' = x - t + p with x = X and t = wY both brought into [0, p)
+// first (the Shoup product accepts any 32-bit Y, so Y needs no correction).
+__device__ __forceinline__ void ct_bfly31(uint32_t &X, uint32_t &Y, uint2 w, uint32_t p) {
+  const uint32_t x = cond_sub(X, p);
+  const uint32_t t = cond_sub(shoup_mul(Y, w.x, w.y, p), p);
+  X = x + t;
+  Y = x - t + p;
+}
+
+// Inverse with twiddle -w: X' = x + y, Y' = (y - x + p) w, x and y the inputs
+// brought into [0, p).
+__device__ __forceinline__ void gs_bfly31(uint32_t &X, uint32_t &Y, uint2 w, uint32_t p) {
+  const uint32_t x = cond_sub(X, p), y = cond_sub(Y, p);
+  X = x + y;
+  Y = shoup_mul(y - x + p, w.x, w.y, p);
+}
+
 // Stage s of the forward transform corrects X when s = 7, 11, 15, ...: the
 // bounds run 2p -> 4p -> .. -> 16p after stage 6, then 10p (corrected),
 // 12p, 14p, 16p, 10p (corrected), ...; 16p < 2^32.
@@ -133,7 +153,7 @@ __device__ __forceinline__ void load_twiddles(const uint2 *__restrict__ tw, uint
   }
 }
 
-template <int LOGN, int E, int NP, int S0, int H, int U>
+template <int LOGN, int E, int NP, int S0, int H, int U, bool P31>
 __device__ __forceinline__ void fwd_stage(uint32_t (&x)[NP][E], const uint2 *__restrict__ tw, uint32_t tau,
                                           uint32_t p, uint32_t two_p, uint32_t eight_p) {
   constexpr uint32_t N = 1u << LOGN;
@@ -153,9 +173,13 @@ __device__ __forceinline__ void fwd_stage(uint32_t (&x)[NP][E], const uint2 *__r
       for (int q = 0; q < (1 << H); ++q) {
         if (q & HALF) continue;
 #pragma unroll
-        for (int k = 0; k < NP; ++k)
-          ct_bfly<CORR>(x[k][b * (1 << H) + q], x[k][b * (1 << H) + q + HALF], w[(b << U) + (q >> (H - U))], p, two_p,
-                        eight_p);
+        for (int k = 0; k < NP; ++k) {
+          if constexpr (P31)
+            ct_bfly31(x[k][b * (1 << H) + q], x[k][b * (1 << H) + q + HALF], w[(b << U) + (q >> (H - U))], p);
+          else
+            ct_bfly<CORR>(x[k][b * (1 << H) + q], x[k][b * (1 << H) + q + HALF], w[(b << U) + (q >> (H - U))], p,
+                          two_p, eight_p);
+        }
       }
   } else {
 #pragma unroll
@@ -166,14 +190,18 @@ __device__ __forceinline__ void fwd_stage(uint32_t (&x)[NP][E], const uint2 *__r
         if (q & HALF) continue;
         const uint2 w = tw[(1u << S) + (g << U) + (q >> (H - U))];
 #pragma unroll
-        for (int k = 0; k < NP; ++k)
-          ct_bfly<CORR>(x[k][b * (1 << H) + q], x[k][b * (1 << H) + q + HALF], w, p, two_p, eight_p);
+        for (int k = 0; k < NP; ++k) {
+          if constexpr (P31)
+            ct_bfly31(x[k][b * (1 << H) + q], x[k][b * (1 << H) + q + HALF], w, p);
+          else
+            ct_bfly<CORR>(x[k][b * (1 << H) + q], x[k][b * (1 << H) + q + HALF], w, p, two_p, eight_p);
+        }
       }
     }
   }
 }
 
-template <int LOGN, int E, int NP, int S0, int H, int U>
+template <int LOGN, int E, int NP, int S0, int H, int U, bool P31>
 __device__ __forceinline__ void inv_stage(uint32_t (&x)[NP][E], const uint2 *__restrict__ tw, uint32_t tau,
                                           uint32_t p, uint32_t eight_p) {
   constexpr bool LAST = (S0 + H == LOGN);  // the pass the inverse starts with
@@ -195,9 +223,13 @@ __device__ __forceinline__ void inv_stage(uint32_t (&x)[NP][E], const uint2 *__r
         if (q & HALF) continue;
         const int idx = CNT - 1 - ((b << U) + (q >> (H - U)));
 #pragma unroll
-        for (int k = 0; k < NP; ++k)
-          gs_bfly(x[k][b * (1 << H) + q], x[k][b * (1 << H) + q + HALF], w[idx], p, eight_p,
-                  inv_corrects<LAST, H, U>(q));
+        for (int k = 0; k < NP; ++k) {
+          if constexpr (P31)
+            gs_bfly31(x[k][b * (1 << H) + q], x[k][b * (1 << H) + q + HALF], w[idx], p);
+          else
+            gs_bfly(x[k][b * (1 << H) + q], x[k][b * (1 << H) + q + HALF], w[idx], p, eight_p,
+                    inv_corrects<LAST, H, U>(q));
+        }
       }
   } else {
 #pragma unroll
@@ -209,25 +241,30 @@ __device__ __forceinline__ void inv_stage(uint32_t (&x)[NP][E], const uint2 *__r
         const uint32_t G = (g << U) + (q >> (H - U));
         const uint2 w = tw[(2u << S) - 1u - G];
 #pragma unroll
-        for (int k = 0; k < NP; ++k)
-          gs_bfly(x[k][b * (1 << H) + q], x[k][b * (1 << H) + q + HALF], w, p, eight_p, inv_corrects<LAST, H, U>(q));
+        for (int k = 0; k < NP; ++k) {
+          if constexpr (P31)
+            gs_bfly31(x[k][b * (1 << H) + q], x[k][b * (1 << H) + q + HALF], w, p);
+          else
+            gs_bfly(x[k][b * (1 << H) + q], x[k][b * (1 << H) + q + HALF], w, p, eight_p,
+                    inv_corrects<LAST, H, U>(q));
+        }
       }
     }
   }
 }
 
-template <int LOGN, int E, int NP, int S0, int H, int U = 0>
+template <int LOGN, int E, int NP, int S0, int H, bool P31, int U = 0>
 __device__ __forceinline__ void fwd_pass(uint32_t (&x)[NP][E], const uint2 *tw, uint32_t tau, uint32_t p,
                                          uint32_t two_p, uint32_t eight_p) {
-  fwd_stage<LOGN, E, NP, S0, H, U>(x, tw, tau, p, two_p, eight_p);
-  if constexpr (U + 1 < H) fwd_pass<LOGN, E, NP, S0, H, U + 1>(x, tw, tau, p, two_p, eight_p);
+  fwd_stage<LOGN, E, NP, S0, H, U, P31>(x, tw, tau, p, two_p, eight_p);
+  if constexpr (U + 1 < H) fwd_pass<LOGN, E, NP, S0, H, P31, U + 1>(x, tw, tau, p, two_p, eight_p);
 }
 
-template <int LOGN, int E, int NP, int S0, int H, int U = H - 1>
+template <int LOGN, int E, int NP, int S0, int H, bool P31, int U = H - 1>
 __device__ __forceinline__ void inv_pass(uint32_t (&x)[NP][E], const uint2 *tw, uint32_t tau, uint32_t p,
                                          uint32_t eight_p) {
-  inv_stage<LOGN, E, NP, S0, H, U>(x, tw, tau, p, eight_p);
-  if constexpr (U > 0) inv_pass<LOGN, E, NP, S0, H, U - 1>(x, tw, tau, p, eight_p);
+  inv_stage<LOGN, E, NP, S0, H, U, P31>(x, tw, tau, p, eight_p);
+  if constexpr (U > 0) inv_pass<LOGN, E, NP, S0, H, P31, U - 1>(x, tw, tau, p, eight_p);
 }
 
 // A pass whose butterfly groups span S elements keeps the data of every run of
@@ -339,31 +376,31 @@ __device__ __forceinline__ void exchange(uint32_t (&x)[NP][E], uint32_t *xb, uin
 
 // Forward transform of NP polynomials held as x[k][e] = element
 // slot_index<LOGN,E,0,RAD>(tau, e) = tau + e*N/E of polynomial k.
-template <int LOGN, int E, int NP, int XBUF, int PASS = 0>
+template <int LOGN, int E, int NP, int XBUF, bool P31 = false, int PASS = 0>
 __device__ __forceinline__ void ntt_forward(uint32_t (&x)[NP][E], const uint2 *tw, uint32_t *xb, uint32_t tau,
                                             uint32_t p) {
   using S = NttShape<LOGN, E>;
   constexpr int S0 = S::RAD * PASS;
   constexpr int H = S::template h<PASS>();
-  fwd_pass<LOGN, E, NP, S0, H>(x, tw, tau, p, 2 * p, 8 * p);
+  fwd_pass<LOGN, E, NP, S0, H, P31>(x, tw, tau, p, 2 * p, 8 * p);
   if constexpr (PASS + 1 < S::NPASS) {
     exchange<LOGN, E, NP, XBUF, S0, H, S0 + S::RAD, S::template h<PASS + 1>()>(x, xb, tau);
-    ntt_forward<LOGN, E, NP, XBUF, PASS + 1>(x, tw, xb, tau, p);
+    ntt_forward<LOGN, E, NP, XBUF, P31, PASS + 1>(x, tw, xb, tau, p);
   }
 }
 
 // Inverse transform (without the N^{-1} factor).  Input: x[k][e] holds
 // bit-reversed position E*tau + e; output: natural position tau + e*N/E.
-template <int LOGN, int E, int NP, int XBUF, int PASS = NttShape<LOGN, E>::NPASS - 1>
+template <int LOGN, int E, int NP, int XBUF, bool P31 = false, int PASS = NttShape<LOGN, E>::NPASS - 1>
 __device__ __forceinline__ void ntt_inverse(uint32_t (&x)[NP][E], const uint2 *tw, uint32_t *xb, uint32_t tau,
                                             uint32_t p) {
   using S = NttShape<LOGN, E>;
   constexpr int S0 = S::RAD * PASS;
   constexpr int H = S::template h<PASS>();
-  inv_pass<LOGN, E, NP, S0, H>(x, tw, tau, p, 8 * p);
+  inv_pass<LOGN, E, NP, S0, H, P31>(x, tw, tau, p, 8 * p);
   if constexpr (PASS > 0) {
     exchange<LOGN, E, NP, XBUF, S0, H, S0 - S::RAD, S::RAD>(x, xb, tau);
-    ntt_inverse<LOGN, E, NP, XBUF, PASS - 1>(x, tw, xb, tau, p);
+    ntt_inverse<LOGN, E, NP, XBUF, P31, PASS - 1>(x, tw, xb, tau, p);
   }
 }
 

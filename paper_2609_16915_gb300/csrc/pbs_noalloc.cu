@@ -92,15 +92,13 @@ extern "C" int rosetta_pbs_batch_noalloc(rosetta_ctx *c, const uint64_t *lwe_in,
   a.lwe_in = lwe_in;
   a.lut = lut;
   a.lwe_big_out = big;
-  a.bsk = c->d_bsk;
-  a.tw = c->d_tw;
+  br_key_args(c, &a);
   a.n = c->prm.lwe_dim;
   a.level = c->prm.pbs_level;
   a.base_log = c->prm.pbs_base_log;
   a.msg_bits = c->prm.msg_bits;
   a.batch = batch;
   a.num_luts = 1;
-  a.cc = c->cc;
   cudaError_t e = launch_blind_rotate(a, c->logN, c->dig16, s);
   if (e != cudaSuccess) return ROSETTA_ERR_CUDA;
 

@@ -52,6 +52,17 @@ double ext_product_bits(const rosetta_params &p) {
   return v + e;
 }
 
+// Does the exact integer value of every external-product coefficient,
+// |X| <= (k+1) l N 2^(beta-1) 2^63, stay within 0.45 of the product of the
+// three 31-bit primes (the margin the three-prime CRT quotient needs)?
+bool fits_three_primes(const rosetta_params &p) {
+  using u128 = unsigned __int128;
+  u128 M3 = 1;
+  for (int q = 0; q < kPrimes31; ++q) M3 *= kPrime31List[q];
+  const u128 bound = (static_cast<u128>(p.glwe_dim + 1) * p.pbs_level * p.poly_size) << (p.pbs_base_log - 1 + 63);
+  return bound * 20 <= M3 * 9;
+}
+
 int check_params(const rosetta_params &p) {
   const uint32_t logN = log2_exact(p.poly_size);
   if (logN < 8 || logN > 13) return ROSETTA_ERR_UNSUPPORTED_PARAMS;
@@ -157,9 +168,7 @@ BrArgs br_args(const rosetta_ctx *c, const uint64_t *in, uint32_t batch, const u
   a.lwe_in = in;
   a.lut = lut;
   a.lwe_big_out = big;
-  a.bsk = c->d_bsk;
-  a.bsk_words = c->bsk_words;
-  a.tw = c->d_tw;
+  br_key_args(c, &a);
   a.n = c->prm.lwe_dim;
   a.level = c->prm.pbs_level;
   a.base_log = c->prm.pbs_base_log;
@@ -167,7 +176,6 @@ BrArgs br_args(const rosetta_ctx *c, const uint64_t *in, uint32_t batch, const u
   a.batch = batch;
   a.num_luts = 1;
   a.err_flag = c->d_err;
-  a.cc = c->cc;
   return a;
 }
 
@@ -298,12 +306,30 @@ int rosetta_params_init(rosetta_ctx **out, const rosetta_params *p, int cuda_dev
   c->logN = logN;
   c->dig16 = dig16;
   std::vector<uint2> tw((size_t)kPrimes << logN);
-  if (!build_tables(logN, tw.data(), &c->cc)) {
+  if (!build_tables(logN, kPrimes, tw.data(), &c->cc)) {
     delete c;
     return ROSETTA_ERR_UNSUPPORTED_PARAMS;
   }
+  // The blind rotation runs over three 31-bit primes where the bound allows
+  // it, the kernel exists for the ring size and level, and two of its CTAs
+  // fit an SM's shared memory; over the four 28-bit primes otherwise.
+  int smem_sm = 0, smem_rsv = 0;
+  cudaDeviceGetAttribute(&smem_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, cuda_device);
+  cudaDeviceGetAttribute(&smem_rsv, cudaDevAttrReservedSharedMemoryPerBlock, cuda_device);
+  const size_t smem3 = br3_smem_bytes(logN, p->pbs_level, p->lwe_dim);
+  std::vector<uint2> tw31;
+  if (fits_three_primes(*p) && br3_supported(logN, p->pbs_level, dig16) && smem3 <= (size_t)max_smem &&
+      2 * (smem3 + (size_t)smem_rsv) <= (size_t)smem_sm) {
+    tw31.resize((size_t)kPrimes31 << logN);
+    if (build_tables(logN, kPrimes31, tw31.data(), &c->cc31)) c->br_primes = kPrimes31;
+  }
   cudaError_t e = cudaMalloc(&c->d_tw, tw.size() * sizeof(uint2));
   if (e == cudaSuccess) e = cudaMemcpy(c->d_tw, tw.data(), tw.size() * sizeof(uint2), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess && c->br_primes == kPrimes31) {
+    e = cudaMalloc(&c->d_tw31, tw31.size() * sizeof(uint2));
+    if (e == cudaSuccess)
+      e = cudaMemcpy(c->d_tw31, tw31.data(), tw31.size() * sizeof(uint2), cudaMemcpyHostToDevice);
+  }
   if (e == cudaSuccess) e = cudaMalloc(&c->d_lut, sizeof(uint64_t) << p->msg_bits);
   if (e == cudaSuccess) e = cudaMalloc(&c->d_err, sizeof(uint32_t));
   if (e == cudaSuccess) e = cudaMemset(c->d_err, 0, sizeof(uint32_t));
@@ -344,20 +370,22 @@ int rosetta_upload_bsk(rosetta_ctx *c, const uint64_t *bsk, size_t n_words, int 
     }
     src = tmp;
   }
-  // one 32-bit residue per prime for every raw word
-  if (!c->d_bsk) e = cudaMalloc(&c->d_bsk, want * kPrimes * sizeof(uint32_t));
+  // one 32-bit residue per prime of the blind rotation's set for every raw word
+  const bool three = c->br_primes == kPrimes31;
+  if (!c->d_bsk) e = cudaMalloc(&c->d_bsk, want * c->br_primes * sizeof(uint32_t));
   if (e != cudaSuccess) {
     if (tmp) cudaFreeAsync(tmp, s);
     return cuda_fail(e);
   }
-  e = launch_bsk_transform(src, c->d_bsk, c->d_tw, c->cc, c->logN, p.lwe_dim, p.pbs_level, s);
+  e = launch_bsk_transform(src, c->d_bsk, three ? c->d_tw31 : c->d_tw, three ? c->cc31 : c->cc, c->logN, p.lwe_dim,
+                           p.pbs_level, c->br_primes, s);
   if (tmp) cudaFreeAsync(tmp, s);
   if (e != cudaSuccess) return cuda_fail(e);
   if (!src_is_device) {
     e = cudaStreamSynchronize(s);  // caller may free the host buffer on return
     if (e != cudaSuccess) return cuda_fail(e);
   }
-  c->bsk_words = want * kPrimes;
+  c->bsk_words = want * c->br_primes;
   c->have_bsk = true;
   return ROSETTA_OK;
 }
@@ -702,6 +730,8 @@ int rosetta_segmented_lookup_batch(rosetta_ctx *c, const uint64_t *glwe_x, const
   return e == cudaSuccess ? ROSETTA_OK : cuda_fail(e);
 }
 
+int rosetta_ntt_primes(const rosetta_ctx *c) { return c ? static_cast<int>(c->br_primes) : ROSETTA_ERR_INVALID_ARG; }
+
 int rosetta_selftest_wait_timeout(rosetta_ctx *c, uint32_t limit_us, void *stream) {
   if (!c || limit_us == 0 || limit_us > 1000000) return ROSETTA_ERR_INVALID_ARG;
   if (cudaSetDevice(c->device) != cudaSuccess) return ROSETTA_ERR_CUDA;
@@ -763,6 +793,7 @@ void rosetta_destroy(rosetta_ctx *c) {
   cudaSetDevice(c->device);
   cudaDeviceSynchronize();
   cudaFree(c->d_tw);
+  cudaFree(c->d_tw31);
   cudaFree(c->d_bsk);
   cudaFree(c->d_ksk);
   cudaFree(c->d_corr);

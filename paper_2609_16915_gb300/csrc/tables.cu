@@ -1,5 +1,6 @@
-// Host-side precomputation: twiddle tables and CRT constants for the four
-// NTT primes.  Runs once per context.
+// Host-side precomputation: twiddle tables and CRT constants for a set of NTT
+// primes (the four 28-bit primes, or the three 31-bit ones).  Runs once per
+// context and set.
 #include <vector>
 
 #include "internal.h"
@@ -60,16 +61,21 @@ uint32_t shoup(uint32_t w, uint32_t p) { return static_cast<uint32_t>((static_ca
 
 }  // namespace
 
-bool build_tables(uint32_t logN, uint2 *tw_host, CrtConsts *cc) {
+bool build_tables(uint32_t logN, uint32_t primes, uint2 *tw_host, CrtConsts *cc) {
   const uint32_t N = 1u << logN;
+  if (primes != kPrimes && primes != kPrimes31) return false;
+  const uint32_t *list = primes == kPrimes ? kPrimeList : kPrime31List;
+  // 28-bit set in (2^28 - 2^18, 2^28): lazy residues up to 16p fit 32 bits and
+  // the CRT quotient may use 2^28 in place of p; 31-bit set in
+  // (2^31 - 2^19, 2^31): residues below 2p fit, the quotient uses 2^31
+  const uint32_t top = primes == kPrimes ? 28 : 31, gap = primes == kPrimes ? 18 : 19;
+  *cc = CrtConsts{};
   u128 M = 1;
-  for (int q = 0; q < kPrimes; ++q) M *= kPrimeList[q];
+  for (uint32_t q = 0; q < primes; ++q) M *= list[q];
   cc->M_mod64 = static_cast<uint64_t>(M);
-  for (int q = 0; q < kPrimes; ++q) {
-    const uint32_t p = kPrimeList[q];
-    // (2^28 - 2^18, 2^28): lazy residues up to 16p fit 32 bits, and the CRT
-    // quotient may use 2^28 in place of p
-    if (!is_prime(p) || (p - 1) % (2 * N) != 0 || p >= (1u << 28) || p <= (1u << 28) - (1u << 18)) return false;
+  for (uint32_t q = 0; q < primes; ++q) {
+    const uint32_t p = list[q];
+    if (!is_prime(p) || (p - 1) % (2 * N) != 0 || p >= (1u << top) || p <= (1u << top) - (1u << gap)) return false;
     const uint32_t g = generator(p);
     if (!g) return false;
     const uint32_t psi = powmod(g, (p - 1) / (2 * N), p);  // primitive 2N-th root of unity

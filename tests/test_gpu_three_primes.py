@@ -1,0 +1,162 @@
+"""The three-prime blind rotation (primes just under 2^31, clusters of three
+CTAs) against the oracle, and the rule that picks it.
+
+A context takes three primes where the external product's bound
+(k+1) l N 2^(beta-1) 2^63 stays within 0.45 of their product, the kernel
+exists (N = 4096, 16-bit digits, l <= 2) and two of its CTAs fit one SM's
+shared memory; four primes otherwise.  The outputs are the same words
+either way, so every case is compared word for word with the oracle: each
+compiled level, the encrypted-test-polynomial variant, many LUTs, the
+largest magnitude the rule admits at this ring size, and the four-prime
+kernels the rule now bypasses at N = 4096."""
+
+import numpy as np
+import pytest
+
+import oracle as O
+import workload as W
+from tests import extreme_util as X
+from tests import gpu_util as G
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2609_16915_gb300 import build
+    build.build()
+
+
+def _params(N, base_log, level, n, batch=3):
+    return W.Params(f"t{N}_{base_log}x{level}_{n}", n=n, k=1, N=N, pbs_base_log=base_log, pbs_level=level,
+                    ks_base_log=4, ks_level=4, msg_bits=3, lwe_sigma_log2=40, glwe_sigma_log2=20,
+                    lut=("square_mod",), msg=("uniform",), batch=batch, seed=N + 7 * base_log + level + n)
+
+
+def _br3_smem(N, level, n):
+    """Shared memory of one three-prime CTA (the kernel's layout)."""
+    T = N // 8
+    b = 8 * N + 48 * T + 48 * T + 4 * (N + N // 8) + 12 * level * T + 2 * (n + 1)
+    return (b + 15) & ~15
+
+
+def _primes(p):
+    import paper_2609_16915_gb300 as R
+    ctx = R.Context(p, device=0)
+    try:
+        return ctx.ntt_primes()
+    finally:
+        ctx.close()
+
+
+@pytest.mark.parametrize("name,want", [("gpt2_mlp", 3), ("standard", 4), ("paper_dims", 4), ("llama_silu", 4),
+                                       ("tiny", 4)])
+def test_named_sets_take_the_expected_prime_set(name, want):
+    """N = 4096 (l = 2, beta = 15: bound 0.25 of the three primes' product)
+    takes three; N = 2048 with beta = 23 needs four (bound above 2^97); the
+    N = 8192 set fits three primes but has no three-prime kernel."""
+    assert _primes(W.CONFIGS[name]) == want
+
+
+def test_rule_at_the_bound_and_at_the_shared_memory_limit():
+    import torch
+    # beta = 16, l = 2 at N = 4096: bound 0.50 of the product, over 0.45
+    assert _primes(_params(4096, 16, 2, 3)) == 4
+    # l = 3, beta = 15: bound 0.375, but its CTA (116 KB) leaves one per SM
+    assert _primes(_params(4096, 15, 3, 3)) == 4
+    # the largest n whose two CTAs fit one SM (2 x (smem + 1 KB reserved))
+    props = torch.cuda.get_device_properties(0)
+    per_sm = getattr(props, "shared_memory_per_multiprocessor", None)
+    if per_sm is None:
+        pytest.skip("this torch does not report shared memory per SM")
+    n_max = max(n for n in range(1, 4096) if 2 * (_br3_smem(4096, 2, n) + 1024) <= per_sm)
+    assert _primes(_params(4096, 15, 2, n_max)) == 3
+    assert _primes(_params(4096, 15, 2, n_max + 1)) == 4
+
+
+@pytest.mark.parametrize("base_log,level", [(16, 1), (12, 1), (15, 2), (12, 2)])
+def test_every_three_prime_level_bitexact(base_log, level):
+    """Dense masks on a short LWE (every CMux step runs), every output word
+    of blind rotation + extraction and of the whole PBS."""
+    p = _params(4096, base_log, level, 4)
+    bsk, ksk = W.uniform_keys(p)
+    lwe = W.uniform_ciphertexts(p, p.batch, sub=3)
+    lut = W.lut_torus(p)
+    ctx = G.make_ctx(p, bsk, ksk)
+    assert ctx.ntt_primes() == 3
+    big = G.gpu_br_extract(ctx, p, lwe, lut)
+    want = O.blind_rotate_extract_batch(p, bsk, lwe, lut)
+    assert np.array_equal(big, want)
+    assert np.array_equal(G.gpu_pbs(ctx, p, lwe, lut), O.keyswitch_batch(p, ksk, want))
+    ctx.close()
+
+
+def test_three_prime_glwe_test_polynomials_and_many_luts():
+    """The per-ciphertext GLWE test polynomial variant and per-ciphertext
+    LUT selection on the three-prime kernel."""
+    p = _params(4096, 15, 2, 3, batch=4)
+    bsk, ksk = W.uniform_keys(p)
+    lwe = W.uniform_ciphertexts(p, p.batch, sub=5)
+    g = np.random.default_rng(77)
+    glwe = g.integers(0, 2**64, size=(p.batch, p.k + 1, p.N), dtype=np.uint64, endpoint=False)
+    ctx = G.make_ctx(p, bsk, ksk)
+    assert ctx.ntt_primes() == 3
+    out = G.empty_dev(p.batch, p.k + 1, p.N)
+    ctx.blind_rotate_glwe_batch(G.to_dev(lwe), G.to_dev(glwe), out)
+    ctx.sync_status()
+    assert np.array_equal(G.to_host(out), O.blind_rotate_glwe_batch(p, bsk, lwe, glwe))
+    luts = np.stack([W.lut_torus(p, codes=[(m * (j + 1) + j) % 8 for m in range(8)]) for j in range(3)])
+    import torch
+    idx = np.array([2, 0, 1, 2])
+    got = G.empty_dev(p.batch, p.n + 1)
+    ctx.pbs_batch_multi_lut(G.to_dev(lwe), G.to_dev(luts), torch.from_numpy(idx.astype(np.int32)).cuda(), got)
+    ctx.sync_status()
+    assert np.array_equal(G.to_host(got), O.pbs_batch_multi_lut(p, bsk, ksk, lwe, luts, idx))
+    ctx.close()
+
+
+@pytest.mark.parametrize("sign", [+1, -1])
+def test_three_prime_product_at_the_largest_admitted_magnitude(sign):
+    """l = 2, beta = 15 at N = 4096: every digit at -B/2 against key words
+    of one sign close to 2^63, so coefficient N-1 sums 4 N terms of one sign,
+    2^91 = 0.25 of the three primes' product (the largest bound among the
+    sets that take three primes at this ring size).  Against the oracle and
+    the closed form."""
+    p = _params(4096, 15, 2, 2, batch=1)
+    bsk, lwe, glwe, C = X.case(p, sign, seed=41)
+    ksk = W.uniform_keys(p)[1]
+    ctx = G.make_ctx(p, bsk, ksk)
+    assert ctx.ntt_primes() == 3
+    out = G.empty_dev(1, p.k + 1, p.N)
+    ctx.blind_rotate_glwe_batch(G.to_dev(lwe), G.to_dev(glwe), out)
+    ctx.sync_status()
+    got = G.to_host(out)
+    assert np.array_equal(got, O.blind_rotate_glwe_batch(p, bsk, lwe, glwe))
+    want, peak = X.expected(p, bsk, C)
+    assert peak > 0.249 * 2**92.999
+    assert [[int(w) for w in row] for row in got[0]] == want
+    ctx.close()
+
+
+@pytest.mark.parametrize("base_log,level,n", [(16, 1, 4700), (16, 2, 4), (15, 3, 4)])
+def test_four_prime_kernels_the_rule_bypasses(base_log, level, n):
+    """The four-prime kernels with 16-bit digits at N = 4096 that the
+    three-prime rule now bypasses: one level only past the shared-memory
+    limit (n = 4700: sparse masks, 12 CMux steps, one at the last index),
+    two levels with beta = 16 (bound over 0.45 of the product), three levels
+    (a three-prime CTA would not fit twice per SM)."""
+    p = _params(4096, base_log, level, n, batch=2)
+    bsk, ksk = W.uniform_keys(p)
+    if n > 100:
+        lwe = G.sparse_lwe(p, p.batch, 12, seed=level)
+        lwe[:, p.n - 1] = np.uint64(3 << 60)
+    else:
+        lwe = W.uniform_ciphertexts(p, p.batch, sub=9)
+    lut = W.lut_torus(p)
+    ctx = G.make_ctx(p, bsk, ksk)
+    assert ctx.ntt_primes() == 4
+    assert np.array_equal(G.gpu_br_extract(ctx, p, lwe, lut), O.blind_rotate_extract_batch(p, bsk, lwe, lut))
+    ctx.close()

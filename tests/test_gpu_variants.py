@@ -2,7 +2,10 @@
 
 The blind-rotation kernel is specialised on the ring size, the digit width
 (16-bit digits when the gadget base is at most 2^16) and, from N = 2048 up,
-the gadget level count (1, 2, 3, or any).  Each case picks a gadget that
+the gadget level count (1, 2, 3, or any).  At N = 4096 the 16-bit-digit
+cases with one or two levels run the three-prime kernel (the context picks
+it where the product's bound allows; tests/test_gpu_three_primes.py also
+reaches the four-prime kernels those cases bypass).  Each case picks a gadget that
 lands on one specialisation the headline parameter sets do not reach; dense
 masks on a short LWE keep the oracle's schoolbook products quick.  Parameter
 sets whose CTA does not fit the shared memory of one SM are refused at

@@ -13,7 +13,13 @@ negacyclic product mod 2^64 (numpy's wrapping uint64 convolution); a
 separate pass propagates worst-case bounds through the same correction
 schedule at every ring size, so the schedule is checked independently of
 the data.  The rules mirror csrc/ntt.cuh, csrc/modarith.cuh and
-csrc/blind_rotate.cu."""
+csrc/blind_rotate.cu.
+
+The three-prime kernel (csrc/blind_rotate3.cu) has its own model below:
+primes just under 2^31, every transform value in [0, 2p), forward outputs
+brought below p before the multiply-accumulate, row pairs accumulated in
+[0, 2p), and the CRT quotient estimated against 2^31; exact up to the
+largest magnitude the context accepts for it (0.45 of the primes' product)."""
 
 import os
 import re
@@ -26,10 +32,20 @@ E, RAD = 8, 3
 M32 = (1 << 32) - 1
 
 
-def primes():
+def _prime_list(name):
     text = open(os.path.join(ROOT, "paper_2609_16915_gb300", "csrc", "internal.h")).read()
-    m = re.search(r"kPrimeList\[kPrimes\]\s*=\s*\{([^}]*)\}", text)
+    m = re.search(name + r"\[\w+\]\s*=\s*\{([^}]*)\}", text)
     return [int(v.strip().rstrip("u")) for v in m.group(1).split(",")]
+
+
+def primes():
+    """The four 28-bit primes of the four-prime kernel."""
+    return _prime_list("kPrimeList")
+
+
+def primes31():
+    """The three 31-bit primes of the three-prime kernel."""
+    return _prime_list("kPrime31List")
 
 
 def generator(p):
@@ -338,3 +354,160 @@ def test_lazy_bounds_hold_in_the_worst_case(L):
     correction."""
     assert worst_case_bounds(L) <= 16
     assert 16 * max(primes()) < 2**32
+
+
+# ---- the three-prime kernel: primes in (2^31 - 2^19, 2^31) ----
+
+def cond(x, b):
+    """min(x, x - b) on 32-bit words: x in [0, 2b) -> [0, b)."""
+    return min(x, (x - b) & M32)
+
+
+def forward31(L, xs, tw, p):
+    """Forward transform with the P31 butterflies: inputs and outputs in [0, 2p)."""
+    ps = passes(L)
+    for pi, (S0, H) in enumerate(ps):
+        for U in range(H):
+            S = S0 + U
+            for tau, i0, i1, G, _ in butterflies(L, S0, H, U):
+                x = xs[tau]
+                X, Y = x[i0], x[i1]
+                assert X < 2 * p and Y < 2 * p
+                w, ws = tw[(1 << S) + G]
+                xr, t = cond(X, p), cond(shoup(Y, w, ws, p), p)
+                assert xr < p and t < p
+                x[i0], x[i1] = (xr + t) & M32, (xr - t + p) & M32
+                assert x[i0] < 2 * p and x[i1] < 2 * p
+        if pi + 1 < len(ps):
+            xs = exchange(L, xs, ps[pi], ps[pi + 1])
+    return xs
+
+
+def inverse31(L, xs, tw, p):
+    """Inverse transform (without N^-1) with the P31 butterflies: [0, 2p) in and out."""
+    ps = passes(L)
+    for pi in range(len(ps) - 1, -1, -1):
+        S0, H = ps[pi]
+        for U in range(H - 1, -1, -1):
+            S = S0 + U
+            for tau, i0, i1, G, _ in butterflies(L, S0, H, U):
+                x = xs[tau]
+                X, Y = x[i0], x[i1]
+                assert X < 2 * p and Y < 2 * p
+                xr, yr = cond(X, p), cond(Y, p)
+                w, ws = tw[(2 << S) - 1 - G]
+                x[i0], x[i1] = xr + yr, shoup((yr - xr + p) & M32, w, ws, p)
+                assert x[i0] < 2 * p and x[i1] < 2 * p
+        if pi > 0:
+            xs = exchange(L, xs, ps[pi], ps[pi - 1])
+    return xs
+
+
+def crt_quotient31(ys):
+    """round(sum y_q / p_q) estimated from the shifted sum against 2^31."""
+    ysum = sum(y >> 3 for y in ys)
+    assert ysum < 2**31
+    return (ysum + (1 << 27)) >> 28
+
+
+def external_product31(L, digits, G, P):
+    """The three-prime kernel's external product (rows in pairs)."""
+    N, R = 1 << L, len(digits)
+    M = 1
+    for p in P:
+        M *= p
+    ys = [[None] * len(P) for _ in range(2)]
+    for qi, p in enumerate(P):
+        assert 2**30 < p < 2**31
+        tw, p_inv = twiddles(L, p), pow(p, -1, 1 << 32)
+        crt_c = pow((M // p) % p, -1, p) * pow(N, -1, p) % p
+        Gh = []
+        for r in range(R):
+            per_c = []
+            for c in range(2):
+                centred = [(w - (1 << 64) if w >= 1 << 63 else w) % p for w in G[r][c]]
+                fk = forward31(L, to_regs(L, centred), tw, p)
+                per_c.append([[cond(v, p) * (1 << 32) % p * crt_c % p for v in row] for row in fk])
+            Gh.append(per_c)
+        oh = None
+        for r0 in range(0, R, 2):
+            fx = [forward31(L, to_regs(L, [(d + p) & M32 for d in digits[r0 + k]]), tw, p) for k in range(2)]
+            acc = [[[0] * E for _ in range(N // E)] for _ in range(2)]
+            for tau in range(N // E):
+                for e in range(E):
+                    x0, x1 = cond(fx[0][tau][e], p), cond(fx[1][tau][e], p)
+                    for c in range(2):
+                        rr = redc(x0 * Gh[r0][c][tau][e] + x1 * Gh[r0 + 1][c][tau][e], p, p_inv)
+                        acc[c][tau][e] = rr if oh is None else cond(oh[c][tau][e], p) + cond(rr, p)
+                        assert acc[c][tau][e] < 2 * p
+            oh = acc
+        for c in range(2):
+            y = from_regs(L, inverse31(L, oh[c], tw, p))
+            assert max(y) < 2 * p
+            ys[c][qi] = y
+    out = []
+    for c in range(2):
+        col = []
+        for j in range(N):
+            yq = [ys[c][qi][j] for qi in range(len(P))]
+            s = sum(y * ((M // p) % 2**64) for y, p in zip(yq, P))
+            col.append((s - crt_quotient31(yq) * (M % 2**64)) % 2**64)
+        out.append(col)
+    return out
+
+
+def test_three_prime_set():
+    """Three primes c 2^14 + 1 in (2^31 - 2^19, 2^31): 2N | p - 1 up to
+    N = 8192, 2p < 2^32, and a product above 2^92.999."""
+    P = primes31()
+    assert len(P) == 3 and len(set(P)) == 3
+    for p in P:
+        assert 2**31 - 2**19 < p < 2**31 and (p - 1) % 2**14 == 0
+        assert p % 2 and all(p % d for d in range(3, int(p**0.5) + 1, 2))  # prime
+    M = P[0] * P[1] * P[2]
+    assert M > 2**92.999
+
+
+def fits_three_primes(k, l, N, beta):
+    """The context's rule: (k+1) l N 2^(beta-1) 2^63 <= 0.45 M3."""
+    P = primes31()
+    return (k + 1) * l * N * 2 ** (beta - 1) * 2**63 * 20 <= P[0] * P[1] * P[2] * 9
+
+
+def test_three_prime_rule_and_quotient_margin():
+    """The N = 4096 set (l = 2, beta = 15) and the N = 8192 one (l = 3,
+    beta = 14) fit three primes, the N = 2048 set (l = 1, beta = 23) and
+    N = 4096 with beta = 16 do not; and for every accepted bound the
+    quotient estimate is off by less than 0.5 - 0.45."""
+    assert fits_three_primes(1, 2, 4096, 15) and fits_three_primes(1, 3, 8192, 14)
+    assert not fits_three_primes(1, 1, 2048, 23) and not fits_three_primes(1, 2, 4096, 16)
+    P = primes31()
+    # undershoot of y/2^31 against y/p for y < 2p, plus the shifted sum's truncation
+    err = sum(2 * (2**31 - p) / 2**31 for p in P) + 3 * 8 / 2**31 + 2**-28
+    assert err < 0.05
+
+
+@pytest.mark.parametrize("L,beta,R", [(8, 15, 4), (9, 16, 2), (10, 14, 6), (12, 15, 4)])
+def test_emulated_three_prime_external_product_is_exact(L, beta, R):
+    N = 1 << L
+    rs = np.random.default_rng(100 + L)
+    half = 1 << (beta - 1)
+    digits = [[int(v) for v in rs.integers(-half, half, N)] for _ in range(R)]
+    digits[0][0], digits[0][1] = -half, half - 1
+    G = [[[int(v) for v in rs.integers(0, 2**64, N, dtype=np.uint64)] for _ in range(2)] for _ in range(R)]
+    G[0][0][0], G[0][0][1] = 1 << 63, (1 << 63) - 1
+    assert external_product31(L, digits, G, primes31()) == expected(digits, G)
+
+
+@pytest.mark.parametrize("L,beta,R", [(12, 15, 4), (12, 15, 6)])
+def test_emulated_three_prime_external_product_at_the_largest_magnitude(L, beta, R):
+    """Every digit -B/2 against every key word -2^63 at N = 4096: coefficient
+    N-1 reaches R N 2^(beta-1) 2^63, 0.25 M3 with two levels (the N = 4096
+    set) and 0.375 M3 with three (the largest bound a three-prime kernel
+    accepts at this ring size)."""
+    N = 1 << L
+    P = primes31()
+    assert R * N * 2 ** (beta - 1) * 2**63 <= 0.38 * P[0] * P[1] * P[2]
+    digits = [[-(1 << (beta - 1))] * N for _ in range(R)]
+    G = [[[1 << 63] * N for _ in range(2)] for _ in range(R)]
+    assert external_product31(L, digits, G, P) == expected(digits, G)

@@ -458,7 +458,18 @@ class _NoClock:
         return None
 
 
-def measure_other_config(name, torch, dev, R, steps, warmup, sms, sm_max, bfly_per_clk):
+def butterfly_rate(rates, primes):
+    """Measured butterflies per clock per SM of the butterfly the blind
+    rotation runs: the lazy one of the 28-bit primes (five instructions) or
+    the one of the 31-bit primes (nine)."""
+    return rates["butterfly_p31"]["per_clk_per_sm"] / 9.0 if primes == 3 else rates["butterfly"]["per_clk_per_sm"] / 5.0
+
+
+def kernel_name(primes):
+    return "blind_rotate3_kernel (3 primes)" if primes == 3 else "blind_rotate_kernel (4 primes)"
+
+
+def measure_other_config(name, torch, dev, R, steps, warmup, sms, sm_max, rates):
     """PBS/s of another parameter set at its full batch (uniform-word keys and
     ciphertexts resident, L2 flushed between steps), the blind rotation timed
     alone, and its fractions of the two peaks."""
@@ -498,13 +509,16 @@ def measure_other_config(name, torch, dev, R, steps, warmup, sms, sm_max, bfly_p
     br_ms = a1.elapsed_time(b1)
     br_ops, _ = int_ops_per_pbs(p)
     achieved = br_ops * batch / (br_ms / 1e3) / 1e12
+    primes = ctx.ntt_primes()
+    bfly_per_clk = butterfly_rate(rates, primes)
     ctx.close()
     del lwe, out, big, flush
     torch.cuda.empty_cache()
     return {"workload": describe(p, batch), "value": batch / (ms / 1e3), "unit": UNIT, "ms_per_step": ms,
-            "steps": steps, "warmup": warmup, "blind_rotation_ms": br_ms, "achieved_tops": achieved,
-            "frac": achieved / (sms * 128 * sm_max * 1e6 / 1e12),
-            "frac_of_butterfly_rate_peak": achieved / (bfly_per_clk * 8 * sms * sm_max * 1e6 / 1e12)}
+            "steps": steps, "warmup": warmup, "kernel": kernel_name(primes), "blind_rotation_ms": br_ms,
+            "achieved_tops": achieved, "frac": achieved / (sms * 128 * sm_max * 1e6 / 1e12),
+            "frac_of_butterfly_rate_peak": achieved / (bfly_per_clk * 8 * sms * sm_max * 1e6 / 1e12),
+            "butterflies_per_clk_per_sm": round(bfly_per_clk, 2)}
 
 
 # ---------------------------------------------------------------------------- GPU arm
@@ -647,7 +661,8 @@ def main():
     # multiply pipe bounds it below the 128-lane issue limit): every counted
     # operation at the rate the butterfly's 8 counted operations run
     rates = measure_int_rates(torch, dev)
-    bfly_per_clk = rates["butterfly"]["per_clk_per_sm"] / 5.0
+    primes = ctx.ntt_primes()
+    bfly_per_clk = butterfly_rate(rates, primes)
     mix_peak = bfly_per_clk * 8 * sms * sm_max * 1e6 / 1e12
     pbs_roof = alu_peak * 1e12 / (br_ops + ks_ops)
     limbs = ks_tensor_limbs(p, batch)
@@ -672,7 +687,7 @@ def main():
         "scaling": "weak", "vs_baseline": None, "dtype": "u64", "data": "synthetic",
         "config": {"workload": describe(p, batch), "batch": batch, "parallelism": f"dp{world}" if world > 1 else "none",
                    "l2": "flushed between steps (256 MB write)", "keys": "uniform words, resident"},
-        "roofline": {"bound": "alu", "kernel": "blind_rotate_kernel", "achieved": achieved, "peak": alu_peak,
+        "roofline": {"bound": "alu", "kernel": kernel_name(primes), "achieved": achieved, "peak": alu_peak,
                      "unit": "Tops/s (int32)", "frac": achieved / alu_peak, "traffic": measured_traffic(p, batch),
                      "peak_basis": f"{sms} SMs x 128 int32 lanes x {sm_max:.0f} MHz (sm_max_mhz of MEASURED_PEAKS.json)",
                      "kernel_ms": br_ms, "keyswitch_ms": ks_ms, "keyswitch": ks_roof,
@@ -693,7 +708,7 @@ def main():
         # steps); uniform-word keys as above
         other = {}
         for name, st, wu in (("gpt2_mlp", 3, 2), ("llama_silu", 2, 1)):
-            other[name] = measure_other_config(name, torch, dev, R, st, wu, sms, sm_max, bfly_per_clk)
+            other[name] = measure_other_config(name, torch, dev, R, st, wu, sms, sm_max, rates)
         ml = run_multi_lut(_Steps(2, 1), p, batch, torch, dev, R, _NoClock)
         other["multi_lut"] = {k: ml[k] for k in ("metric", "value", "unit", "ms_per_step", "steps")}
         other["multi_lut"]["workload"] = ml["config"]["workload"]

@@ -47,9 +47,22 @@ struct Br3Shape {
   static constexpr int T = N / E;  // threads per CTA
   static constexpr int LOG_T = LOGN - 3;
   // resident CTAs per SM the register allocation must allow (2 x 112 KB of
-  // shared memory at N = 4096)
+  // shared memory at N = 4096, 1 x 198 KB at 8192)
   static constexpr int MIN_CTAS = LOGN <= 12 ? 2 : 1;
+  // At N = 8192 the digits and the received residues share one region (the
+  // CTA would need 234 KB otherwise): one more cluster barrier per step, after
+  // the last digit gather, keeps a push from overwriting digits still unread.
+  static constexpr bool SHARED_DIG_RES = LOGN >= 13;
 };
+
+// 32-bit words of the digit and residue region: residues [2][T][4] + [2][T][2],
+// digits [l][T][2] + [l][T]
+__host__ __device__ constexpr size_t br3_res_words(size_t T) { return 12 * T; }
+__host__ __device__ constexpr size_t br3_dig_words(size_t T, size_t level) { return 3 * level * T; }
+__host__ __device__ constexpr size_t br3_region_words(size_t T, size_t level, bool shared) {
+  return shared ? (br3_res_words(T) > br3_dig_words(T, level) ? br3_res_words(T) : br3_dig_words(T, level))
+                : br3_res_words(T) + br3_dig_words(T, level);
+}
 
 __device__ __forceinline__ uint32_t pack16(int32_t lo, int32_t hi) {
   return (static_cast<uint32_t>(lo) & 0xFFFFu) | (static_cast<uint32_t>(hi) << 16);
@@ -62,16 +75,17 @@ __device__ __forceinline__ int32_t hi16(uint32_t w) { return static_cast<int16_t
 // Shared memory, in this order (16-byte aligned pieces):
 //   tw    uint2  [N]           twiddles of prime `rank`
 //   acc   uint64 [2][3][T]     owned accumulator words (component, slot, thread)
+//   xb    uint32 [N + N/8]     transform exchange buffer
 //   res4  uint32 [2][T][4]     residues from the two other primes: slots 0, 1 of both components
 //   res2  uint32 [2][T][2]     slot 2 of both components (owners 0 and 1)
-//   xb    uint32 [N + N/8]     transform exchange buffer
 //   dig8  uint32 [l][T][2]     16-bit digits of each row pair: slots 0, 1 of both rows
 //   dig4  uint32 [l][T]        slot 2 of both rows (owners 0 and 1)
 //   atil  uint16 [n+1]         switched mask and body
+// (at N = 8192 dig8 and dig4 start where res4 starts)
 size_t br3_smem_bytes(uint32_t logN, uint32_t level, uint32_t n) {
   const size_t N = size_t(1) << logN, T = N / 8;
-  size_t b = N * sizeof(uint2) + 6 * T * sizeof(uint64_t) + 2 * T * 6 * sizeof(uint32_t) +
-             (N + N / 8) * sizeof(uint32_t) + level * T * 3 * sizeof(uint32_t) + (n + 1) * sizeof(uint16_t);
+  size_t b = N * sizeof(uint2) + 6 * T * sizeof(uint64_t) + (N + N / 8) * sizeof(uint32_t) +
+             br3_region_words(T, level, logN >= 13) * sizeof(uint32_t) + (n + 1) * sizeof(uint16_t);
   return (b + 15) & ~size_t(15);
 }
 
@@ -90,14 +104,15 @@ __global__ void __launch_bounds__(Br3Shape<LOGN>::T, Br3Shape<LOGN>::MIN_CTAS) b
   if (!dbg_ok(ct < a.batch, a.err_flag)) return;  // the whole cluster shares ct
 
   extern __shared__ __align__(16) unsigned char smem[];
+  constexpr bool SHARED = B::SHARED_DIG_RES;
   uint2 *tw = reinterpret_cast<uint2 *>(smem);
   uint64_t *acc = reinterpret_cast<uint64_t *>(tw + N);
-  uint32_t *res4 = reinterpret_cast<uint32_t *>(acc + 6 * T);
+  uint32_t *xb = reinterpret_cast<uint32_t *>(acc + 6 * T);
+  uint32_t *res4 = xb + S::XB_WORDS;
   uint32_t *res2 = res4 + 2 * T * 4;
-  uint32_t *xb = res2 + 2 * T * 2;
-  uint32_t *dig8 = xb + S::XB_WORDS;
+  uint32_t *dig8 = SHARED ? res4 : res2 + 2 * T * 2;
   uint32_t *dig4 = dig8 + L * T * 2;
-  uint16_t *atil = reinterpret_cast<uint16_t *>(dig4 + L * T);
+  uint16_t *atil = reinterpret_cast<uint16_t *>(res4 + br3_region_words(T, L, SHARED));
 
   const uint32_t p = a.cc.pr[rank].p;
   const uint32_t p_inv = a.cc.pr[rank].p_inv;
@@ -240,6 +255,9 @@ __global__ void __launch_bounds__(Br3Shape<LOGN>::T, Br3Shape<LOGN>::MIN_CTAS) b
           x[1][q + 2] = static_cast<uint32_t>(hi16(w4)) + p;
         }
       }
+      if constexpr (SHARED) {
+        if (P == L - 1) cluster.sync();  // every digit read: the region may now take residues
+      }
       ntt_forward<LOGN, E, 2, 1, true>(x, tw, xb, tau, p);  // outputs in [0, 2p)
       // below p, so that a row pair's two products sum below 2 p^2 < p 2^32
 #pragma unroll
@@ -342,10 +360,13 @@ __global__ void __launch_bounds__(Br3Shape<LOGN>::T, Br3Shape<LOGN>::MIN_CTAS) b
   cluster.sync();
 }
 
-// Three levels would need 116 KB per CTA at N = 4096: one CTA per SM, where
-// the four-prime kernel keeps two; so one or two levels only.
+// Compiled: N = 4096 with one or two levels (three would need 116 KB per CTA,
+// one per SM where the four-prime kernel keeps two), N = 8192 with one to
+// three.  The context also checks that the CTAs fit as densely as the
+// four-prime kernel's.
 bool br3_supported(uint32_t logN, uint32_t level, bool dig16) {
-  return dig16 && logN == 12 && level >= 1 && level <= 2;
+  if (!dig16 || level < 1) return false;
+  return (logN == 12 && level <= 2) || (logN == 13 && level <= 3);
 }
 
 template <int LOGN, int LEV>
@@ -372,11 +393,12 @@ static cudaError_t launch_br3_t(const BrArgs &a, cudaStream_t s) {
 }
 
 cudaError_t launch_blind_rotate3(const BrArgs &a, uint32_t logN, cudaStream_t s) {
-  if (a.primes != kPrimes31 || logN != 12) return cudaErrorInvalidValue;
+  if (a.primes != kPrimes31 || !br3_supported(logN, a.level, true)) return cudaErrorInvalidValue;
+  if (logN == 12) return a.level == 1 ? launch_br3_t<12, 1>(a, s) : launch_br3_t<12, 2>(a, s);
   switch (a.level) {
-    case 1: return launch_br3_t<12, 1>(a, s);
-    case 2: return launch_br3_t<12, 2>(a, s);
-    default: return cudaErrorInvalidValue;
+    case 1: return launch_br3_t<13, 1>(a, s);
+    case 2: return launch_br3_t<13, 2>(a, s);
+    default: return launch_br3_t<13, 3>(a, s);
   }
 }
 

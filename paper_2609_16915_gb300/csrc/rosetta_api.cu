@@ -311,15 +311,18 @@ int rosetta_params_init(rosetta_ctx **out, const rosetta_params *p, int cuda_dev
     return ROSETTA_ERR_UNSUPPORTED_PARAMS;
   }
   // The blind rotation runs over three 31-bit primes where the bound allows
-  // it, the kernel exists for the ring size and level, and two of its CTAs
-  // fit an SM's shared memory; over the four 28-bit primes otherwise.
+  // it, the kernel exists for the ring size and level, and as many of its
+  // CTAs fit an SM's shared memory as of the four-prime kernel's; over the
+  // four 28-bit primes otherwise.
   int smem_sm = 0, smem_rsv = 0;
   cudaDeviceGetAttribute(&smem_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, cuda_device);
   cudaDeviceGetAttribute(&smem_rsv, cudaDevAttrReservedSharedMemoryPerBlock, cuda_device);
   const size_t smem3 = br3_smem_bytes(logN, p->pbs_level, p->lwe_dim);
+  const size_t smem4 = br_smem_bytes(logN, p->pbs_level, p->lwe_dim, dig16);
+  const auto per_sm = [&](size_t b) { return (size_t)smem_sm / (b + (size_t)smem_rsv); };
   std::vector<uint2> tw31;
   if (fits_three_primes(*p) && br3_supported(logN, p->pbs_level, dig16) && smem3 <= (size_t)max_smem &&
-      2 * (smem3 + (size_t)smem_rsv) <= (size_t)smem_sm) {
+      per_sm(smem3) >= per_sm(smem4)) {
     tw31.resize((size_t)kPrimes31 << logN);
     if (build_tables(logN, kPrimes31, tw31.data(), &c->cc31)) c->br_primes = kPrimes31;
   }

@@ -3,12 +3,13 @@ CTAs) against the oracle, and the rule that picks it.
 
 A context takes three primes where the external product's bound
 (k+1) l N 2^(beta-1) 2^63 stays within 0.45 of their product, the kernel
-exists (N = 4096, 16-bit digits, l <= 2) and two of its CTAs fit one SM's
-shared memory; four primes otherwise.  The outputs are the same words
-either way, so every case is compared word for word with the oracle: each
-compiled level, the encrypted-test-polynomial variant, many LUTs, the
-largest magnitude the rule admits at this ring size, and the four-prime
-kernels the rule now bypasses at N = 4096."""
+exists (16-bit digits; N = 4096 with l <= 2, N = 8192 with l <= 3) and as
+many of its CTAs fit one SM's shared memory as of the four-prime kernel's;
+four primes otherwise.  The outputs are the same words either way, so every
+case is compared word for word with the oracle: each compiled ring size and
+level, the encrypted-test-polynomial variant, many LUTs, the largest
+magnitude the rule admits at each ring size, and the four-prime kernels the
+rule now bypasses at N = 4096."""
 
 import numpy as np
 import pytest
@@ -37,9 +38,18 @@ def _params(N, base_log, level, n, batch=3):
 
 
 def _br3_smem(N, level, n):
-    """Shared memory of one three-prime CTA (the kernel's layout)."""
+    """Shared memory of one three-prime CTA (the kernel's layout; digits and
+    residues share one region at N = 8192)."""
     T = N // 8
-    b = 8 * N + 48 * T + 48 * T + 4 * (N + N // 8) + 12 * level * T + 2 * (n + 1)
+    region = max(12 * T, 3 * level * T) if N >= 8192 else 12 * T + 3 * level * T
+    b = 8 * N + 48 * T + 4 * (N + N // 8) + 4 * region + 2 * (n + 1)
+    return (b + 15) & ~15
+
+
+def _br4_smem(N, level, n):
+    """Shared memory of one four-prime CTA with 16-bit digits (N >= 2048)."""
+    Q = N // 4
+    b = 8 * N + 16 * Q + 32 * Q + 4 * (N + N // 8) + 4 * level * Q + 2 * (n + 1)
     return (b + 15) & ~15
 
 
@@ -52,12 +62,13 @@ def _primes(p):
         ctx.close()
 
 
-@pytest.mark.parametrize("name,want", [("gpt2_mlp", 3), ("standard", 4), ("paper_dims", 4), ("llama_silu", 4),
+@pytest.mark.parametrize("name,want", [("gpt2_mlp", 3), ("llama_silu", 3), ("standard", 4), ("paper_dims", 4),
                                        ("tiny", 4)])
 def test_named_sets_take_the_expected_prime_set(name, want):
     """N = 4096 (l = 2, beta = 15: bound 0.25 of the three primes' product)
-    takes three; N = 2048 with beta = 23 needs four (bound above 2^97); the
-    N = 8192 set fits three primes but has no three-prime kernel."""
+    and N = 8192 (l = 3, beta = 14: 0.375) take three; N = 2048 with
+    beta = 23 needs four (bound above 2^97); N = 256 has no three-prime
+    kernel."""
     assert _primes(W.CONFIGS[name]) == want
 
 
@@ -67,21 +78,27 @@ def test_rule_at_the_bound_and_at_the_shared_memory_limit():
     assert _primes(_params(4096, 16, 2, 3)) == 4
     # l = 3, beta = 15: bound 0.375, but its CTA (116 KB) leaves one per SM
     assert _primes(_params(4096, 15, 3, 3)) == 4
-    # the largest n whose two CTAs fit one SM (2 x (smem + 1 KB reserved))
+    # three primes only while their CTAs fit an SM as densely as the four-prime
+    # kernel's (1 KB reserved per CTA): both two per SM up to some n, then two
+    # against one, then one each
     props = torch.cuda.get_device_properties(0)
     per_sm = getattr(props, "shared_memory_per_multiprocessor", None)
     if per_sm is None:
         pytest.skip("this torch does not report shared memory per SM")
-    n_max = max(n for n in range(1, 4096) if 2 * (_br3_smem(4096, 2, n) + 1024) <= per_sm)
-    assert _primes(_params(4096, 15, 2, n_max)) == 3
-    assert _primes(_params(4096, 15, 2, n_max + 1)) == 4
+    fits = lambda b: per_sm // (b + 1024)
+    rule = [fits(_br3_smem(4096, 2, n)) >= fits(_br4_smem(4096, 2, n)) for n in range(1, 6000)]
+    flips = [n for n in range(2, 6000) if rule[n - 1] != rule[n - 2]]
+    assert rule[0] and len(flips) == 2, flips          # e.g. [1536, 3584] on a 228 KB SM
+    for n in sorted({flips[0] - 1, flips[0], flips[1] - 1, flips[1], 5999}):
+        assert _primes(_params(4096, 15, 2, n)) == (3 if rule[n - 1] else 4), n
 
 
-@pytest.mark.parametrize("base_log,level", [(16, 1), (12, 1), (15, 2), (12, 2)])
-def test_every_three_prime_level_bitexact(base_log, level):
+@pytest.mark.parametrize("N,base_log,level", [(4096, 16, 1), (4096, 12, 1), (4096, 15, 2), (4096, 12, 2),
+                                              (8192, 15, 1), (8192, 14, 2), (8192, 14, 3), (8192, 11, 3)])
+def test_every_three_prime_level_bitexact(N, base_log, level):
     """Dense masks on a short LWE (every CMux step runs), every output word
     of blind rotation + extraction and of the whole PBS."""
-    p = _params(4096, base_log, level, 4)
+    p = _params(N, base_log, level, 4 if N == 4096 else 2, batch=3 if N == 4096 else 2)
     bsk, ksk = W.uniform_keys(p)
     lwe = W.uniform_ciphertexts(p, p.batch, sub=3)
     lut = W.lut_torus(p)
@@ -94,10 +111,11 @@ def test_every_three_prime_level_bitexact(base_log, level):
     ctx.close()
 
 
-def test_three_prime_glwe_test_polynomials_and_many_luts():
+@pytest.mark.parametrize("N,base_log,level", [(4096, 15, 2), (8192, 14, 3)])
+def test_three_prime_glwe_test_polynomials_and_many_luts(N, base_log, level):
     """The per-ciphertext GLWE test polynomial variant and per-ciphertext
     LUT selection on the three-prime kernel."""
-    p = _params(4096, 15, 2, 3, batch=4)
+    p = _params(N, base_log, level, 3 if N == 4096 else 2, batch=4)
     bsk, ksk = W.uniform_keys(p)
     lwe = W.uniform_ciphertexts(p, p.batch, sub=5)
     g = np.random.default_rng(77)
@@ -118,14 +136,16 @@ def test_three_prime_glwe_test_polynomials_and_many_luts():
     ctx.close()
 
 
+@pytest.mark.parametrize("N,base_log,level,share", [(4096, 15, 2, 0.249), (8192, 14, 3, 0.374)])
 @pytest.mark.parametrize("sign", [+1, -1])
-def test_three_prime_product_at_the_largest_admitted_magnitude(sign):
-    """l = 2, beta = 15 at N = 4096: every digit at -B/2 against key words
-    of one sign close to 2^63, so coefficient N-1 sums 4 N terms of one sign,
-    2^91 = 0.25 of the three primes' product (the largest bound among the
-    sets that take three primes at this ring size).  Against the oracle and
-    the closed form."""
-    p = _params(4096, 15, 2, 2, batch=1)
+def test_three_prime_product_at_the_largest_admitted_magnitude(N, base_log, level, share, sign):
+    """Every digit at -B/2 against key words of one sign close to 2^63, so
+    coefficient N-1 sums 2 l N terms of one sign: 2^91 = 0.25 of the three
+    primes' product with l = 2, beta = 15 at N = 4096, 3 x 2^91 = 0.375 with
+    l = 3, beta = 14 at N = 8192 (the largest bounds among the sets that take
+    three primes at these ring sizes).  Against the oracle and the closed
+    form."""
+    p = _params(N, base_log, level, 2, batch=1)
     bsk, lwe, glwe, C = X.case(p, sign, seed=41)
     ksk = W.uniform_keys(p)[1]
     ctx = G.make_ctx(p, bsk, ksk)
@@ -136,7 +156,7 @@ def test_three_prime_product_at_the_largest_admitted_magnitude(sign):
     got = G.to_host(out)
     assert np.array_equal(got, O.blind_rotate_glwe_batch(p, bsk, lwe, glwe))
     want, peak = X.expected(p, bsk, C)
-    assert peak > 0.249 * 2**92.999
+    assert peak > share * 2**92.999
     assert [[int(w) for w in row] for row in got[0]] == want
     ctx.close()
 

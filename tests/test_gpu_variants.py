@@ -2,10 +2,12 @@
 
 The blind-rotation kernel is specialised on the ring size, the digit width
 (16-bit digits when the gadget base is at most 2^16) and, from N = 2048 up,
-the gadget level count (1, 2, 3, or any).  At N = 4096 the 16-bit-digit
-cases with one or two levels run the three-prime kernel (the context picks
-it where the product's bound allows; tests/test_gpu_three_primes.py also
-reaches the four-prime kernels those cases bypass).  Each case picks a gadget that
+the gadget level count (1, 2, 3, or any).  At N = 4096 and 8192 the
+16-bit-digit cases whose product bound is small enough run the three-prime
+kernel (the context picks it where the bound allows; (4096, 16, 2),
+(8192, 15, 2), (8192, 16, 1) and (8192, 16, 3) stay on four primes, and
+tests/test_gpu_three_primes.py reaches the other four-prime kernels those
+cases bypass).  Each case picks a gadget that
 lands on one specialisation the headline parameter sets do not reach; dense
 masks on a short LWE keep the oracle's schoolbook products quick.  Parameter
 sets whose CTA does not fit the shared memory of one SM are refused at
@@ -45,7 +47,7 @@ VARIANTS = [
     (256, 24, 2), (512, 28, 1), (1024, 8, 6),
     (2048, 16, 1), (2048, 13, 2), (2048, 11, 3), (2048, 16, 4), (2048, 28, 1), (2048, 24, 2), (2048, 21, 3),
     (4096, 16, 1), (4096, 12, 2), (4096, 11, 3), (4096, 9, 5), (4096, 28, 1), (4096, 24, 2), (4096, 21, 3),
-    (8192, 16, 1), (8192, 10, 2), (8192, 16, 3), (8192, 28, 1),
+    (8192, 16, 1), (8192, 10, 2), (8192, 15, 2), (8192, 16, 3), (8192, 28, 1),
 ]
 
 

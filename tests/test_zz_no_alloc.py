@@ -85,3 +85,29 @@ def test_noalloc_rejects_oversize_and_host_buffers(setup):
     assert _call_noalloc(R, small, big[:2], lut, out[:2]) == 0
     small.sync_status(stream=0)
     small.close()
+
+
+def test_noalloc_on_a_three_prime_context(setup):
+    """The N = 4096 set runs the three-prime kernel: the same words as
+    rosetta_pbs_batch and, at a dense and a sparse position, as the oracle."""
+    R, G, _, _ = setup
+    p = W.CONFIGS["gpt2_mlp"]
+    bsk, ksk = W.uniform_keys(p, seed=23)
+    ctx = G.make_ctx(p, bsk, ksk)
+    assert ctx.ntt_primes() == 3
+    lut_h = W.lut_torus(p)
+    lut = G.to_dev(lut_h)
+    lwe_h = W.uniform_ciphertexts(p, 40, sub=34)
+    lwe_h[[39]] = G.sparse_lwe(p, 1, 5, seed=35)
+    lwe = G.to_dev(lwe_h)
+    want = G.empty_dev(40, p.n + 1)
+    ctx.pbs_batch(lwe, lut, want, stream=0)
+    ctx.sync_status(stream=0)
+    got = G.empty_dev(40, p.n + 1)
+    assert _call_noalloc(R, ctx, lwe, lut, got) == 0
+    ctx.sync_status(stream=0)
+    got_h = G.to_host(got)
+    assert np.array_equal(got_h, G.to_host(want))
+    pos = np.array([7, 39])
+    assert np.array_equal(got_h[pos], O.pbs_batch(p, bsk, ksk, lwe_h[pos], lut_h))
+    ctx.close()

@@ -107,11 +107,10 @@ int rosetta_params_init(rosetta_ctx **out, const rosetta_params *p, int cuda_dev
  * product over: 4 (primes just below 2^28, one CTA per prime in a cluster of
  * four) or 3 (primes just below 2^31, a cluster of three).  The context takes
  * three where (k+1) l N 2^(beta-1) 2^63 <= 0.45 x 2^92.999 (the three primes'
- * product), a three-prime kernel exists (beta <= 16; N = 4096 with l <= 2 or
- * N = 8192 with l <= 3) and as many of its CTAs fit one SM's shared memory as
- * of the four-prime kernel's (on a 228 KB SM at N = 4096, l = 2: n <= 1535,
- * two CTAs per SM each, or n >= 3584, one each); e.g. N = 4096, l = 2,
- * beta = 15 and N = 8192, l = 3, beta = 14.  Either way the outputs are the same words: the product is
+ * product), a three-prime kernel exists (beta <= 16, N = 4096 or 8192,
+ * l <= 3) and as many of its CTAs fit one SM's shared memory as of the
+ * four-prime kernel's (always the case at N = 4096: its CTA is the smaller);
+ * e.g. N = 4096, l = 2, beta = 15 and N = 8192, l = 3, beta = 14.  Either way the outputs are the same words: the product is
  * exact.  Fixed at rosetta_params_init.  Returns 3 or 4, or INVALID_ARG for a
  * NULL context. */
 int rosetta_ntt_primes(const rosetta_ctx *ctx);

@@ -19,7 +19,8 @@
 //     them as acc[component][slot h][thread tau];
 //   * the residue exchange: a prime-CTA keeps the residues of its own slots in
 //     registers across the cluster barrier (its threads are their owners) and
-//     sends every other owner its slots, one packed group per thread.
+//     leaves every other owner's slots, one packed group per thread, in its
+//     own exchange buffer, from which the owners read them in phase 3.
 // Per ciphertext and step the cluster runs 3 (l + 1) x 2 transforms instead
 // of 4 (l + 1) x 2, each about 15 % dearer in butterfly instructions.
 #include <cooperative_groups.h>
@@ -46,23 +47,13 @@ struct Br3Shape {
   static constexpr int E = 8;
   static constexpr int T = N / E;  // threads per CTA
   static constexpr int LOG_T = LOGN - 3;
-  // resident CTAs per SM the register allocation must allow (2 x 112 KB of
+  // resident CTAs per SM the register allocation must allow (2 x 92-98 KB of
   // shared memory at N = 4096, 1 x 198 KB at 8192)
   static constexpr int MIN_CTAS = LOGN <= 12 ? 2 : 1;
-  // At N = 8192 the digits and the received residues share one region (the
-  // CTA would need 234 KB otherwise): one more cluster barrier per step, after
-  // the last digit gather, keeps a push from overwriting digits still unread.
-  static constexpr bool SHARED_DIG_RES = LOGN >= 13;
+  // exchange buffer words: N + N/8 for the transforms, extended to 12 T so
+  // that it holds the outgoing residues afterwards
+  static constexpr int XB_WORDS = 12 * T;
 };
-
-// 32-bit words of the digit and residue region: residues [2][T][4] + [2][T][2],
-// digits [l][T][2] + [l][T]
-__host__ __device__ constexpr size_t br3_res_words(size_t T) { return 12 * T; }
-__host__ __device__ constexpr size_t br3_dig_words(size_t T, size_t level) { return 3 * level * T; }
-__host__ __device__ constexpr size_t br3_region_words(size_t T, size_t level, bool shared) {
-  return shared ? (br3_res_words(T) > br3_dig_words(T, level) ? br3_res_words(T) : br3_dig_words(T, level))
-                : br3_res_words(T) + br3_dig_words(T, level);
-}
 
 __device__ __forceinline__ uint32_t pack16(int32_t lo, int32_t hi) {
   return (static_cast<uint32_t>(lo) & 0xFFFFu) | (static_cast<uint32_t>(hi) << 16);
@@ -75,17 +66,17 @@ __device__ __forceinline__ int32_t hi16(uint32_t w) { return static_cast<int16_t
 // Shared memory, in this order (16-byte aligned pieces):
 //   tw    uint2  [N]           twiddles of prime `rank`
 //   acc   uint64 [2][3][T]     owned accumulator words (component, slot, thread)
-//   xb    uint32 [N + N/8]     transform exchange buffer
-//   res4  uint32 [2][T][4]     residues from the two other primes: slots 0, 1 of both components
-//   res2  uint32 [2][T][2]     slot 2 of both components (owners 0 and 1)
+//   xb    uint32 [12 T]        transform exchange buffer (N + N/8 words); after the
+//                              inverse transforms the outgoing residues: [2 other
+//                              owners][T][4] (slots 0, 1 of both components), then
+//                              [2][T][2] (slot 2, owners 0 and 1)
 //   dig8  uint32 [l][T][2]     16-bit digits of each row pair: slots 0, 1 of both rows
 //   dig4  uint32 [l][T]        slot 2 of both rows (owners 0 and 1)
 //   atil  uint16 [n+1]         switched mask and body
-// (at N = 8192 dig8 and dig4 start where res4 starts)
 size_t br3_smem_bytes(uint32_t logN, uint32_t level, uint32_t n) {
   const size_t N = size_t(1) << logN, T = N / 8;
-  size_t b = N * sizeof(uint2) + 6 * T * sizeof(uint64_t) + (N + N / 8) * sizeof(uint32_t) +
-             br3_region_words(T, level, logN >= 13) * sizeof(uint32_t) + (n + 1) * sizeof(uint16_t);
+  size_t b = N * sizeof(uint2) + 6 * T * sizeof(uint64_t) + (12 * T + 3 * level * T) * sizeof(uint32_t) +
+             (n + 1) * sizeof(uint16_t);
   return (b + 15) & ~size_t(15);
 }
 
@@ -104,15 +95,13 @@ __global__ void __launch_bounds__(Br3Shape<LOGN>::T, Br3Shape<LOGN>::MIN_CTAS) b
   if (!dbg_ok(ct < a.batch, a.err_flag)) return;  // the whole cluster shares ct
 
   extern __shared__ __align__(16) unsigned char smem[];
-  constexpr bool SHARED = B::SHARED_DIG_RES;
+  static_assert(B::XB_WORDS >= S::XB_WORDS, "exchange buffer");
   uint2 *tw = reinterpret_cast<uint2 *>(smem);
   uint64_t *acc = reinterpret_cast<uint64_t *>(tw + N);
   uint32_t *xb = reinterpret_cast<uint32_t *>(acc + 6 * T);
-  uint32_t *res4 = xb + S::XB_WORDS;
-  uint32_t *res2 = res4 + 2 * T * 4;
-  uint32_t *dig8 = SHARED ? res4 : res2 + 2 * T * 2;
+  uint32_t *dig8 = xb + B::XB_WORDS;
   uint32_t *dig4 = dig8 + L * T * 2;
-  uint16_t *atil = reinterpret_cast<uint16_t *>(res4 + br3_region_words(T, L, SHARED));
+  uint16_t *atil = reinterpret_cast<uint16_t *>(dig4 + L * T);
 
   const uint32_t p = a.cc.pr[rank].p;
   const uint32_t p_inv = a.cc.pr[rank].p_inv;
@@ -169,7 +158,7 @@ __global__ void __launch_bounds__(Br3Shape<LOGN>::T, Br3Shape<LOGN>::MIN_CTAS) b
   cluster.sync();
 
   const uint32_t acc_s = smem_addr(acc), dig8_s = smem_addr(dig8), dig4_s = smem_addr(dig4);
-  const uint32_t res4_s = smem_addr(res4), res2_s = smem_addr(res2);
+  const uint32_t xb_s = smem_addr(xb);
   const uint32_t bits = a.base_log * L;
   const uint64_t Bmask = (1ull << a.base_log) - 1;
   const uint64_t Bhalf = 1ull << (a.base_log - 1);
@@ -255,9 +244,6 @@ __global__ void __launch_bounds__(Br3Shape<LOGN>::T, Br3Shape<LOGN>::MIN_CTAS) b
           x[1][q + 2] = static_cast<uint32_t>(hi16(w4)) + p;
         }
       }
-      if constexpr (SHARED) {
-        if (P == L - 1) cluster.sync();  // every digit read: the region may now take residues
-      }
       ntt_forward<LOGN, E, 2, 1, true>(x, tw, xb, tau, p);  // outputs in [0, 2p)
       // below p, so that a row pair's two products sum below 2 p^2 < p 2^32
 #pragma unroll
@@ -286,16 +272,18 @@ __global__ void __launch_bounds__(Br3Shape<LOGN>::T, Br3Shape<LOGN>::MIN_CTAS) b
       }
     }
     ntt_inverse<LOGN, E, 2, 1, true>(oh, tw, xb, tau, p);  // outputs in [0, 2p)
-    // CRT-scaled residues (the keys carry the CRT factor): the other owners'
-    // slots are sent, one packed group per owner; the own slots stay here
+    // CRT-scaled residues (the keys carry the CRT factor): one packed group
+    // per other owner, left in this CTA's exchange buffer (once every thread
+    // has finished the transforms' last exchange) at the owner's index among
+    // the other two; the own slots stay in registers
+    __syncthreads();
 #pragma unroll
     for (int o = 0; o < 3; ++o) {
       if (static_cast<uint32_t>(o) == rank) continue;
       const uint32_t q = own_s0(o);
-      const uint32_t ri = rank < static_cast<uint32_t>(o) ? rank : rank - 1;  // remote slot at owner o
-      dsmem_st_v4_u32(dsmem_map(res4_s + (ri * T + tau) * 16u, o),
-                      make_uint4(oh[0][q], oh[0][q + 1], oh[1][q], oh[1][q + 1]));
-      if (o < 2) dsmem_st_v2_u32(dsmem_map(res2_s + (ri * T + tau) * 8u, o), make_uint2(oh[0][q + 2], oh[1][q + 2]));
+      const uint32_t oi = static_cast<uint32_t>(o) < rank ? o : o - 1;  // owner o among the other two
+      *reinterpret_cast<uint4 *>(xb + (oi * T + tau) * 4) = make_uint4(oh[0][q], oh[0][q + 1], oh[1][q], oh[1][q + 1]);
+      if (o < 2) *reinterpret_cast<uint2 *>(xb + 8 * T + (oi * T + tau) * 2) = make_uint2(oh[0][q + 2], oh[1][q + 2]);
     }
     uint32_t yo[2][3];
 #pragma unroll
@@ -308,17 +296,20 @@ __global__ void __launch_bounds__(Br3Shape<LOGN>::T, Br3Shape<LOGN>::MIN_CTAS) b
 
     // ---- phase 3: explicit CRT of the owned slots, accumulate ----
     {
-      const uint4 ra = *reinterpret_cast<const uint4 *>(res4 + tau * 4);
-      const uint4 rb = *reinterpret_cast<const uint4 *>(res4 + (T + tau) * 4);
+      // the two other primes (producers), and this owner's index among the
+      // other two owners of each; their residue groups read remotely
+      const uint32_t q_r0 = rank == 0 ? 1u : 0u, q_r1 = rank == 2 ? 1u : 2u;
+      const uint32_t oa = rank < q_r0 ? rank : rank - 1, ob = rank < q_r1 ? rank : rank - 1;
+      const uint32_t pa = dsmem_map(xb_s, q_r0), pb = dsmem_map(xb_s, q_r1);
+      const uint4 ra = dsmem_ld_v4_u32(pa + (oa * T + tau) * 16u);
+      const uint4 rb = dsmem_ld_v4_u32(pb + (ob * T + tau) * 16u);
       uint2 sa = make_uint2(0u, 0u), sb = make_uint2(0u, 0u);
       if (three) {
-        sa = *reinterpret_cast<const uint2 *>(res2 + tau * 2);
-        sb = *reinterpret_cast<const uint2 *>(res2 + (T + tau) * 2);
+        sa = dsmem_ld_v2_u32(pa + 32u * T + (oa * T + tau) * 8u);
+        sb = dsmem_ld_v2_u32(pb + 32u * T + (ob * T + tau) * 8u);
       }
       const uint32_t y1[2][3] = {{ra.x, ra.y, sa.x}, {ra.z, ra.w, sa.y}};
       const uint32_t y2[2][3] = {{rb.x, rb.y, sb.x}, {rb.z, rb.w, sb.y}};
-      // primes of the residues received in remote slots 0 and 1
-      const uint32_t q_r0 = rank == 0 ? 1u : 0u, q_r1 = rank == 2 ? 1u : 2u;
       const uint64_t m0 = a.cc.pr[rank].Mp_mod64, m1 = a.cc.pr[q_r0].Mp_mod64, m2 = a.cc.pr[q_r1].Mp_mod64;
 #pragma unroll
       for (int c = 0; c < 2; ++c)
@@ -360,13 +351,10 @@ __global__ void __launch_bounds__(Br3Shape<LOGN>::T, Br3Shape<LOGN>::MIN_CTAS) b
   cluster.sync();
 }
 
-// Compiled: N = 4096 with one or two levels (three would need 116 KB per CTA,
-// one per SM where the four-prime kernel keeps two), N = 8192 with one to
-// three.  The context also checks that the CTAs fit as densely as the
-// four-prime kernel's.
+// Compiled: N = 4096 and 8192 with one to three levels.  The context also
+// checks that the CTAs fit an SM as densely as the four-prime kernel's.
 bool br3_supported(uint32_t logN, uint32_t level, bool dig16) {
-  if (!dig16 || level < 1) return false;
-  return (logN == 12 && level <= 2) || (logN == 13 && level <= 3);
+  return dig16 && (logN == 12 || logN == 13) && level >= 1 && level <= 3;
 }
 
 template <int LOGN, int LEV>
@@ -394,7 +382,13 @@ static cudaError_t launch_br3_t(const BrArgs &a, cudaStream_t s) {
 
 cudaError_t launch_blind_rotate3(const BrArgs &a, uint32_t logN, cudaStream_t s) {
   if (a.primes != kPrimes31 || !br3_supported(logN, a.level, true)) return cudaErrorInvalidValue;
-  if (logN == 12) return a.level == 1 ? launch_br3_t<12, 1>(a, s) : launch_br3_t<12, 2>(a, s);
+  if (logN == 12) {
+    switch (a.level) {
+      case 1: return launch_br3_t<12, 1>(a, s);
+      case 2: return launch_br3_t<12, 2>(a, s);
+      default: return launch_br3_t<12, 3>(a, s);
+    }
+  }
   switch (a.level) {
     case 1: return launch_br3_t<13, 1>(a, s);
     case 2: return launch_br3_t<13, 2>(a, s);

@@ -3,8 +3,8 @@ CTAs) against the oracle, and the rule that picks it.
 
 A context takes three primes where the external product's bound
 (k+1) l N 2^(beta-1) 2^63 stays within 0.45 of their product, the kernel
-exists (16-bit digits; N = 4096 with l <= 2, N = 8192 with l <= 3) and as
-many of its CTAs fit one SM's shared memory as of the four-prime kernel's;
+exists (16-bit digits, N = 4096 or 8192, l <= 3) and as many of its CTAs
+fit one SM's shared memory as of the four-prime kernel's;
 four primes otherwise.  The outputs are the same words either way, so every
 case is compared word for word with the oracle: each compiled ring size and
 level, the encrypted-test-polynomial variant, many LUTs, the largest
@@ -38,11 +38,11 @@ def _params(N, base_log, level, n, batch=3):
 
 
 def _br3_smem(N, level, n):
-    """Shared memory of one three-prime CTA (the kernel's layout; digits and
-    residues share one region at N = 8192)."""
+    """Shared memory of one three-prime CTA (the kernel's layout: twiddles,
+    owned accumulator words, the exchange buffer extended to 12 T words for
+    the outgoing residues, packed digits, the switched mask)."""
     T = N // 8
-    region = max(12 * T, 3 * level * T) if N >= 8192 else 12 * T + 3 * level * T
-    b = 8 * N + 48 * T + 4 * (N + N // 8) + 4 * region + 2 * (n + 1)
+    b = 8 * N + 48 * T + 4 * (12 * T + 3 * level * T) + 2 * (n + 1)
     return (b + 15) & ~15
 
 
@@ -76,24 +76,25 @@ def test_rule_at_the_bound_and_at_the_shared_memory_limit():
     import torch
     # beta = 16, l = 2 at N = 4096: bound 0.50 of the product, over 0.45
     assert _primes(_params(4096, 16, 2, 3)) == 4
-    # l = 3, beta = 15: bound 0.375, but its CTA (116 KB) leaves one per SM
-    assert _primes(_params(4096, 15, 3, 3)) == 4
+    assert _primes(_params(4096, 15, 3, 3)) == 3                  # 0.375
     # three primes only while their CTAs fit an SM as densely as the four-prime
-    # kernel's (1 KB reserved per CTA): both two per SM up to some n, then two
-    # against one, then one each
+    # kernel's (1 KB reserved per CTA): the rule at every n up to 12000, and
+    # the context's choice at the ends and around every change
     props = torch.cuda.get_device_properties(0)
     per_sm = getattr(props, "shared_memory_per_multiprocessor", None)
     if per_sm is None:
         pytest.skip("this torch does not report shared memory per SM")
     fits = lambda b: per_sm // (b + 1024)
-    rule = [fits(_br3_smem(4096, 2, n)) >= fits(_br4_smem(4096, 2, n)) for n in range(1, 6000)]
-    flips = [n for n in range(2, 6000) if rule[n - 1] != rule[n - 2]]
-    assert rule[0] and len(flips) == 2, flips          # e.g. [1536, 3584] on a 228 KB SM
-    for n in sorted({flips[0] - 1, flips[0], flips[1] - 1, flips[1], 5999}):
-        assert _primes(_params(4096, 15, 2, n)) == (3 if rule[n - 1] else 4), n
+    for N, beta, level in ((4096, 15, 2), (8192, 14, 3)):
+        top = 12000 if N == 4096 else 3583                        # the four-prime kernel's own n limit
+        rule = [fits(_br3_smem(N, level, n)) >= fits(_br4_smem(N, level, n)) for n in range(1, top + 1)]
+        flips = [n for n in range(2, top + 1) if rule[n - 1] != rule[n - 2]]
+        for n in sorted({1, top} | {m for f in flips for m in (f - 1, f)}):
+            assert _primes(_params(N, beta, level, n)) == (3 if rule[n - 1] else 4), (N, n)
 
 
 @pytest.mark.parametrize("N,base_log,level", [(4096, 16, 1), (4096, 12, 1), (4096, 15, 2), (4096, 12, 2),
+                                              (4096, 15, 3), (4096, 11, 3),
                                               (8192, 15, 1), (8192, 14, 2), (8192, 14, 3), (8192, 11, 3)])
 def test_every_three_prime_level_bitexact(N, base_log, level):
     """Dense masks on a short LWE (every CMux step runs), every output word
@@ -136,15 +137,15 @@ def test_three_prime_glwe_test_polynomials_and_many_luts(N, base_log, level):
     ctx.close()
 
 
-@pytest.mark.parametrize("N,base_log,level,share", [(4096, 15, 2, 0.249), (8192, 14, 3, 0.374)])
+@pytest.mark.parametrize("N,base_log,level,share", [(4096, 15, 3, 0.374), (8192, 14, 3, 0.374)])
 @pytest.mark.parametrize("sign", [+1, -1])
 def test_three_prime_product_at_the_largest_admitted_magnitude(N, base_log, level, share, sign):
     """Every digit at -B/2 against key words of one sign close to 2^63, so
-    coefficient N-1 sums 2 l N terms of one sign: 2^91 = 0.25 of the three
-    primes' product with l = 2, beta = 15 at N = 4096, 3 x 2^91 = 0.375 with
-    l = 3, beta = 14 at N = 8192 (the largest bounds among the sets that take
-    three primes at these ring sizes).  Against the oracle and the closed
-    form."""
+    coefficient N-1 sums 2 l N terms of one sign: 3 x 2^90 = 0.375 of the
+    three primes' product with l = 3, beta = 15 at N = 4096, 3 x 2^91 = 0.375
+    with l = 3, beta = 14 at N = 8192 (the largest bounds among the sets
+    that take three primes at these ring sizes).  Against the oracle and the
+    closed form."""
     p = _params(N, base_log, level, 2, batch=1)
     bsk, lwe, glwe, C = X.case(p, sign, seed=41)
     ksk = W.uniform_keys(p)[1]
@@ -161,13 +162,15 @@ def test_three_prime_product_at_the_largest_admitted_magnitude(N, base_log, leve
     ctx.close()
 
 
-@pytest.mark.parametrize("base_log,level,n", [(16, 1, 4700), (16, 2, 4), (15, 3, 4)])
+@pytest.mark.parametrize("base_log,level,n", [(16, 2, 4), (16, 3, 4), (16, 2, 5000)])
 def test_four_prime_kernels_the_rule_bypasses(base_log, level, n):
     """The four-prime kernels with 16-bit digits at N = 4096 that the
-    three-prime rule now bypasses: one level only past the shared-memory
-    limit (n = 4700: sparse masks, 12 CMux steps, one at the last index),
-    two levels with beta = 16 (bound over 0.45 of the product), three levels
-    (a three-prime CTA would not fit twice per SM)."""
+    three-prime rule leaves to sets whose bound exceeds 0.45 of the three
+    primes' product: two and three levels with beta = 16 (bounds 0.50 and
+    0.75), also at n = 5000 (one CTA per SM; sparse masks, 12 CMux steps, one
+    at the last index).  With one level and beta <= 16 the bound is at most
+    0.25 and the CTA no larger than the four-prime one: every such set takes
+    three primes."""
     p = _params(4096, base_log, level, n, batch=2)
     bsk, ksk = W.uniform_keys(p)
     if n > 100:

@@ -4,10 +4,9 @@ The blind-rotation kernel is specialised on the ring size, the digit width
 (16-bit digits when the gadget base is at most 2^16) and, from N = 2048 up,
 the gadget level count (1, 2, 3, or any).  At N = 4096 and 8192 the
 16-bit-digit cases whose product bound is small enough run the three-prime
-kernel (the context picks it where the bound allows; (4096, 16, 2),
-(8192, 15, 2), (8192, 16, 1) and (8192, 16, 3) stay on four primes, and
-tests/test_gpu_three_primes.py reaches the other four-prime kernels those
-cases bypass).  Each case picks a gadget that
+kernel (the context picks it where the bound allows; (8192, 15, 2),
+(8192, 16, 1) and (8192, 16, 3) stay on four primes, and
+tests/test_gpu_three_primes.py reaches the four-prime kernels at N = 4096).  Each case picks a gadget that
 lands on one specialisation the headline parameter sets do not reach; dense
 masks on a short LWE keep the oracle's schoolbook products quick.  Parameter
 sets whose CTA does not fit the shared memory of one SM are refused at

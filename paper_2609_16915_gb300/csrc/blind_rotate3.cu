@@ -22,7 +22,8 @@
 //     leaves every other owner's slots, one packed group per thread, in its
 //     own exchange buffer, from which the owners read them in phase 3.
 // Per ciphertext and step the cluster runs 3 (l + 1) x 2 transforms instead
-// of 4 (l + 1) x 2, each about 15 % dearer in butterfly instructions.
+// of 4 (l + 1) x 2; a butterfly is seven instructions instead of five and,
+// measured alone, about 15 % slower.
 #include <cooperative_groups.h>
 
 #include "check.cuh"

@@ -33,12 +33,20 @@ def main():
     cs = G.make_ctx(ps, bsk, ksk)
     res["standard_bitexact"] = bool(np.array_equal(G.gpu_pbs(cs, ps, sl, W.lut_torus(ps)),
                                                    O.pbs_batch(ps, bsk, ksk, sl, W.lut_torus(ps))))
-    ctx.selftest_bounds()
-    try:
-        ctx.sync_status()
-        res["bounds_status"] = 0
-    except R.RosettaError as e:
-        res["bounds_status"] = e.status
+    # the three-prime kernel (N = 4096 set) under the same checks
+    pg = W.CONFIGS["gpt2_mlp"]
+    bg, kg = W.uniform_keys(pg, seed=65)
+    gl = G.sparse_lwe(pg, 2, 3, seed=66)
+    cg = G.make_ctx(pg, bg, kg)
+    res["three_prime_bitexact"] = bool(cg.ntt_primes() == 3 and np.array_equal(
+        G.gpu_pbs(cg, pg, gl, W.lut_torus(pg)), O.pbs_batch(pg, bg, kg, gl, W.lut_torus(pg))))
+    for name, c in (("bounds_status", ctx), ("three_prime_bounds_status", cg)):
+        c.selftest_bounds()
+        try:
+            c.sync_status()
+            res[name] = 0
+        except R.RosettaError as e:
+            res[name] = e.status
     # reported once; the context keeps working
     res["after_bitexact"] = bool(np.array_equal(G.gpu_pbs(ctx, p, lwe, lut), O.pbs_batch(p, keys.bsk, keys.ksk, lwe, lut)))
     print(json.dumps(res), flush=True)

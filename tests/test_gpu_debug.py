@@ -31,7 +31,8 @@ def test_debug_build_bitexact_and_reports_bounds():
                        timeout=900)
     assert r.returncode == 0, r.stderr[-3000:]
     res = json.loads(r.stdout.strip().splitlines()[-1])
-    assert res == {"tiny_bitexact": True, "standard_bitexact": True, "bounds_status": -7, "after_bitexact": True}
+    assert res == {"tiny_bitexact": True, "standard_bitexact": True, "three_prime_bitexact": True, "bounds_status": -7,
+                   "three_prime_bounds_status": -7, "after_bitexact": True}
 
 
 def test_regular_build_has_no_bounds_checks():

@@ -183,3 +183,26 @@ def test_four_prime_kernels_the_rule_bypasses(base_log, level, n):
     assert ctx.ntt_primes() == 4
     assert np.array_equal(G.gpu_br_extract(ctx, p, lwe, lut), O.blind_rotate_extract_batch(p, bsk, lwe, lut))
     ctx.close()
+
+
+def test_three_prime_bad_lut_index_is_reported_not_followed():
+    """An out-of-range LUT index on the three-prime kernel: that ciphertext
+    takes LUT 0, the others their own, and the next rosetta_sync_status
+    reports INVALID_ARG once."""
+    import torch
+    import paper_2609_16915_gb300 as R
+    p = _params(4096, 15, 2, 3, batch=3)
+    bsk, ksk = W.uniform_keys(p)
+    lwe = W.uniform_ciphertexts(p, p.batch, sub=8)
+    luts = np.stack([W.lut_torus(p), W.lut_torus(p, codes=[(5 * m + 1) % 8 for m in range(8)])])
+    idx = np.array([1, 7, 0])
+    ctx = G.make_ctx(p, bsk, ksk)
+    assert ctx.ntt_primes() == 3
+    out = G.empty_dev(p.batch, p.n + 1)
+    ctx.pbs_batch_multi_lut(G.to_dev(lwe), G.to_dev(luts), torch.from_numpy(idx.astype(np.int32)).cuda(), out)
+    with pytest.raises(R.RosettaError) as e:
+        ctx.sync_status()
+    assert e.value.status == -1
+    ctx.sync_status()                                    # reported once
+    assert np.array_equal(G.to_host(out), O.pbs_batch_multi_lut(p, bsk, ksk, lwe, luts, np.array([1, 0, 0])))
+    ctx.close()

@@ -511,3 +511,95 @@ def test_emulated_three_prime_external_product_at_the_largest_magnitude(L, beta,
     digits = [[-(1 << (beta - 1))] * N for _ in range(R)]
     G = [[[1 << 63] * N for _ in range(2)] for _ in range(R)]
     assert external_product31(L, digits, G, P) == expected(digits, G)
+
+
+# ---- the exchange buffer's padded layout ----
+
+def xb_pad(kind, i):
+    """The kernels' padding, 4 words after every 32 (kind 0); kind 1, 2 words
+    after every 16, is the alternative the last test measures."""
+    return i + ((i >> 5) << 2) if kind == 0 else i + ((i >> 4) << 1)
+
+
+def pass_accesses(L, S0, H, kind):
+    """Per warp and access instruction, the word addresses each thread
+    touches (one for a scalar access; 4 or 2 consecutive words for the last
+    pass's vector accesses), as the kernel computes them: a per-thread
+    padded base plus a padded compile-time offset."""
+    N, T = 1 << L, (1 << L) // E
+    SIG, SPAN = N >> (S0 + H), N >> S0
+    out = []
+    for warp in range(max(1, T // 32)):
+        ts = range(warp * 32, min(T, warp * 32 + 32))
+        if SIG == 1:
+            width = 4 if kind == 0 else 2
+            for k in range(E // width):
+                acc = []
+                for t in ts:
+                    base = xb_pad(kind, E * t)
+                    assert xb_pad(kind, E * t + k * width) == base + k * width, "additive padding"
+                    assert base % width == 0, "vector alignment"
+                    acc.append([base + k * width + j for j in range(width)])
+                out.append((width, acc))
+        else:
+            for q in range(E):
+                acc = []
+                for t in ts:
+                    pos = (t // SIG) * SPAN + t % SIG
+                    a = xb_pad(kind, pos) + xb_pad(kind, q * SIG)
+                    assert a == xb_pad(kind, pos + q * SIG), "additive padding"
+                    acc.append([a])
+                out.append((1, acc))
+    return out
+
+
+def worst_bank_load(L, S0, H, kind):
+    """Largest number of distinct words one bank serves in one warp access
+    of the pass, over the ideal (1 per scalar access; 32 x width / 32 for
+    vector accesses of `width` words)."""
+    worst = 0
+    for width, acc in pass_accesses(L, S0, H, kind):
+        banks = {}
+        for words in acc:
+            for w in words:
+                banks.setdefault(w % 32, set()).add(w)
+        ideal = max(1, len(acc) * width // 32) if width > 1 else 1
+        worst = max(worst, max(len(v) for v in banks.values()) / ideal)
+    return worst
+
+
+@pytest.mark.parametrize("L", range(8, 14))
+def test_exchange_layout_in_bounds_bijective_and_nearly_conflict_free(L):
+    """Every exchange of the transforms at every ring size: both passes'
+    addresses are the same bijection of the N positions into N + N/8 words
+    (additive in base and offset, vector accesses aligned), and every warp
+    access is free of bank conflicts except in the one pass whose blocks
+    have stride 2 (N = 1024 and 8192), which is two-way conflicted."""
+    N = 1 << L
+    ps = passes(L)
+    for A, B in zip(ps, ps[1:]):
+        kind = 0
+        for S0, H in (A, B):
+            SIG, SPAN = N >> (S0 + H), N >> S0
+            seen = {}
+            for t in range(N // E):
+                for e in range(E):
+                    pos = (t * E + e) if SIG == 1 else (t // SIG) * SPAN + t % SIG + e * SIG
+                    seen[xb_pad(kind, pos)] = pos
+            assert len(seen) == N and max(seen) < N + N // 8
+            expect = 2 if (N >> (S0 + H)) == 2 else 1
+            assert worst_bank_load(L, S0, H, kind) == expect, (L, (S0, H))
+
+
+@pytest.mark.parametrize("L", [10, 13])
+def test_alternative_padding_removes_the_stride_2_conflicts(L):
+    """2 pad words after every 16 serves both passes of the two exchanges
+    around the stride-2 pass without conflicts, but only with 8-byte vector
+    accesses in the last pass (it breaks the 16-byte alignment).  Measured
+    on the N = 8192 set it was 2.8 % slower (twice the last pass's
+    accesses), so the kernels keep the single padding."""
+    N = 1 << L
+    ps = passes(L)
+    k = [i for i, (S0, H) in enumerate(ps) if (N >> (S0 + H)) == 2][0]
+    for S0, H in ps[k - 1:k + 2]:
+        assert worst_bank_load(L, S0, H, 1) == 1

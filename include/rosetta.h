@@ -97,10 +97,12 @@ typedef struct {
  * not fit the four NTT primes: log2((k+1) l N 2^(beta-1) 2^63) + 1 must not
  * exceed 111 (their product is about 2^111.99); and when one blind-rotation
  * CTA (a quarter of the ring) does not fit the device's shared memory per
- * block: 20N + 4.5N per exchange buffer (two for N <= 1024, else one) +
- * l N x {1 for beta <= 16 | 2} + 2(n+1) bytes, which on a 227 KB device
- * admits, at N = 8192, l <= 3 with beta <= 16 (n <= 3583) or l = 1 with
- * beta > 16.  Errors: INVALID_ARG (NULL), UNSUPPORTED_PARAMS, CUDA, OOM. */
+ * block: 12N + max(8N, 4.5N per exchange buffer (two for N <= 1024, else
+ * one)) + l N x {1 for beta <= 16 | 2} + 2(n+1) bytes, which on a 227 KB
+ * device admits at N = 8192, for example, l = 3 with beta <= 16 up to
+ * n = 22015, l = 4 or l = 2 with beta > 16 up to n = 17919, and l = 3 with
+ * beta > 16 up to n = 9727.  Errors: INVALID_ARG (NULL), UNSUPPORTED_PARAMS,
+ * CUDA, OOM. */
 int rosetta_params_init(rosetta_ctx **out, const rosetta_params *p, int cuda_device);
 
 /* Number of NTT primes the context's blind rotation computes the external
@@ -109,8 +111,9 @@ int rosetta_params_init(rosetta_ctx **out, const rosetta_params *p, int cuda_dev
  * three where (k+1) l N 2^(beta-1) 2^63 <= 0.45 x 2^92.999 (the three primes'
  * product), a three-prime kernel exists (beta <= 16, N = 4096 or 8192,
  * l <= 3) and as many of its CTAs fit one SM's shared memory as of the
- * four-prime kernel's (always the case at N = 4096: its CTA is the smaller);
- * e.g. N = 4096, l = 2, beta = 15 and N = 8192, l = 3, beta = 14.  Either way the outputs are the same words: the product is
+ * four-prime kernel's (on a 228 KB SM at N = 4096, l = 2: all n but 10752 to
+ * 12799; at N = 8192, l = 3: n <= 15871); e.g. N = 4096, l = 2, beta = 15
+ * and N = 8192, l = 3, beta = 14.  Either way the outputs are the same words: the product is
  * exact.  Fixed at rosetta_params_init.  Returns 3 or 4, or INVALID_ARG for a
  * NULL context. */
 int rosetta_ntt_primes(const rosetta_ctx *ctx);

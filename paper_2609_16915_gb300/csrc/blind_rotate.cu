@@ -25,11 +25,14 @@
 //   2. each prime-CTA gathers all digits (one vector DSMEM load per owner
 //      and thread), runs forward NTTs two polynomials at a time, multiplies
 //      by the transform-domain BSK_i (streamed from global memory with
-//      16-byte loads, Montgomery form), runs the two inverse NTTs and sends
-//      each owner the CRT-scaled residues of its quarter (one vector DSMEM
-//      store per owner and thread);
-//   3. each owner combines the four residues of its coefficients (explicit
-//      CRT) and adds the result to the accumulator.
+//      16-byte loads, Montgomery form), runs the two inverse NTTs and leaves
+//      the CRT-scaled residues of each owner's quarter in its own exchange
+//      buffer (one vector store per owner and thread);
+//   3. each owner reads the four residues of its coefficients from the four
+//      prime-CTAs (one vector DSMEM load each), combines them (explicit CRT)
+//      and adds the result to the accumulator.
+// Every cross-CTA read follows a write to the writer's own shared memory, so
+// the step's barriers order shared memory only (cluster_sync_shared).
 #include <cooperative_groups.h>
 
 #include <type_traits>
@@ -45,6 +48,14 @@ namespace cg = cooperative_groups;
 // One exchange buffer per polynomial of a pair only where shared memory is
 // plentiful; larger rings share one buffer to keep more CTAs resident.
 __host__ __device__ constexpr int br_xbuf(int logN) { return logN <= 10 ? 2 : 1; }
+
+// Exchange-buffer words: the transforms' XBUF x (N + N/8), and at least 2N
+// (16 T) for the outgoing residues, four groups of four words per thread.
+__host__ __device__ constexpr int br_xb_words(int logN) {
+  return br_xbuf(logN) * ((1 << logN) + (1 << logN) / 8) > 2 * (1 << logN)
+             ? br_xbuf(logN) * ((1 << logN) + (1 << logN) / 8)
+             : 2 * (1 << logN);
+}
 
 // Values per thread in the transforms.  16 halves the CTA-wide exchanges but
 // also the warps per SM; measured on GB300 it is slower at every ring size
@@ -62,7 +73,7 @@ struct BrShape {
   static constexpr int QE = E / 4;                     // first-pass slots per owner quarter
   static constexpr int XBUF = br_xbuf(LOGN);            // exchange buffers (polys)
   // resident CTAs per SM the register allocation must allow (shared memory
-  // allows the same: 4 x 55 KB at N = 2048, 2 x 108 KB at 4096)
+  // allows the same: 4 x 46 KB at N = 2048, 2 x 90 KB at 4096)
   static constexpr int MIN_CTAS = (LOGN <= 11) ? 4 : (LOGN == 12 ? 2 : 1);
 };
 
@@ -86,9 +97,11 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
   extern __shared__ __align__(16) unsigned char smem[];
   uint2 *tw = reinterpret_cast<uint2 *>(smem);                   // [N]
   uint64_t *acc = reinterpret_cast<uint64_t *>(tw + N);          // [2][Q]
-  uint32_t *res = reinterpret_cast<uint32_t *>(acc + 2 * Q);     // [4 primes][T][2 comp][QE halves]
-  uint32_t *xb = res + kPrimes * 2 * Q;                          // [XBUF][XB_WORDS]
-  DigT *dig = reinterpret_cast<DigT *>(xb + B::XBUF * S::XB_WORDS);  // [l row pairs][T][2][QE]
+  // [XBUF][XB_WORDS] for the transforms; after the inverse transforms the
+  // outgoing residues [owner][T][2 comp][QE halves]
+  uint32_t *xb = reinterpret_cast<uint32_t *>(acc + 2 * Q);
+  static_assert(br_xb_words(LOGN) >= B::XBUF * S::XB_WORDS, "exchange buffer");
+  DigT *dig = reinterpret_cast<DigT *>(xb + br_xb_words(LOGN));  // [l row pairs][T][2][QE]
   const uint32_t level = LEV > 0 ? static_cast<uint32_t>(LEV) : a.level;
   uint16_t *atil = reinterpret_cast<uint16_t *>(dig + 2 * level * Q);  // [n+1]
 
@@ -147,7 +160,7 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
 
   // 32-bit shared-memory addresses; mapa turns them into the same location
   // in another CTA of the cluster
-  const uint32_t acc_s = smem_addr(acc), dig_s = smem_addr(dig), res_s = smem_addr(res);
+  const uint32_t acc_s = smem_addr(acc), dig_s = smem_addr(dig), xb_s = smem_addr(xb);
   const uint32_t L2 = 2 * level;
   const uint32_t bits = a.base_log * level;
   const uint64_t Bmask = (1ull << a.base_log) - 1;
@@ -158,13 +171,14 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
   // Packed exchange layouts.  Owner thread tau holds the items (c, jl) =
   // (m / QE, tau + (m % QE) T), m < ITEMS = 2 QE, and prime thread tau needs
   // from owner o exactly the coefficients tau + h T (h < QE) of both
-  // components: so digits are stored as [row pair][tau][row parity][h] and
-  // residues as [prime][tau][component][h], and every transfer between a
-  // pair of threads is one 2 QE-word vector access.
+  // components: so digits are stored as [row pair][tau][row parity][h] in
+  // their owner and residues as [owner][tau][component][h] in their
+  // prime-CTA, and every transfer between a pair of threads is one 2 QE-word
+  // vector access.
   static_assert(ITEMS == 2 * QE, "one packed group of 2 QE items per thread");
   constexpr uint32_t GRP = 2 * QE;  // words per packed group
   const uint32_t dig_t = dig_s + tau * GRP * static_cast<uint32_t>(sizeof(DigT));
-  const uint32_t res_t = res_s + (rank * T + tau) * GRP * 4u;
+  const uint32_t res_t = xb_s + (rank * T + tau) * GRP * 4u;  // this owner's group in every prime-CTA
   // With one gadget level and N <= 2048 the remote bases of this thread's
   // digit and residue groups in each CTA are kept across the steps (measured
   // 1.5 % faster at N = 2048); elsewhere the registers are needed for the
@@ -234,7 +248,7 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
                                                      static_cast<uint32_t>(grp[P][2]), static_cast<uint32_t>(grp[P][3]));
       }
     }
-    cluster.sync();
+    cluster_sync_shared();
 
     // ---- phase 2: transforms and pointwise products for prime `rank` ----
     uint32_t oh[2][E];
@@ -242,14 +256,11 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
     const uint32_t *gbase = a.bsk + (static_cast<size_t>(i) * kPrimes + rank) * kblk;
     const bool key_ok = dbg_ok(a.bsk_words == 0 || (static_cast<size_t>(i) * kPrimes + rank + 1) * kblk <= a.bsk_words,
                                a.err_flag);
-    // Two gadget levels: both row pairs unrolled (no loop-carried register
-    // copies; measured 2.2 % faster at N = 4096, 16-bit digits).  Three levels,
-    // 32-bit digits and N = 8192 keep the loop: unrolled those spill
-    // (three levels at N = 8192: +10 %).
-    constexpr bool PAIR_UNROLLED = (LEV == 2 && LOGN <= 12 && DIG16);
-    constexpr int PAIR_UNROLL = PAIR_UNROLLED ? 2 : 1;
-#pragma unroll PAIR_UNROLL
-    for (uint32_t r0 = 0; r0 < (PAIR_UNROLLED ? 4u : L2); r0 += 2) {
+    // The row pairs stay a rolled loop: unrolled, two levels at N = 4096
+    // spill 56 bytes per thread (pulled residues hold more registers across
+    // phase 2) and three levels at N = 8192 were 10 % slower.
+#pragma unroll 1
+    for (uint32_t r0 = 0; r0 < L2; r0 += 2) {
       // first-pass slot q of thread tau is coefficient tau + q N/E, owned by
       // CTA o = q / QE at local index tau + (q % QE) T: one packed group of
       // the row pair per owner
@@ -311,6 +322,7 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
       }
     }
     ntt_inverse<LOGN, E, 2, B::XBUF>(oh, tw, xb, tau, p);
+    __syncthreads();  // every exchange read done: the buffer takes the outgoing residues
     // CRT-scaled residues (< 8p; the keys carry the CRT factor), one packed
     // group (component, h) per owner
 #pragma unroll
@@ -321,16 +333,16 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
       for (int c = 0; c < 2; ++c)
 #pragma unroll
         for (int h = 0; h < QE; ++h) y[c * QE + h] = oh[c][o * QE + h];
-      dsmem_st_v4_u32(HOIST ? res_r[o] : dsmem_map(res_t, o), make_uint4(y[0], y[1], y[2], y[3]));
+      *reinterpret_cast<uint4 *>(xb + (o * T + tau) * GRP) = make_uint4(y[0], y[1], y[2], y[3]);
     }
-    cluster.sync();
+    cluster_sync_shared();
 
     // ---- phase 3: explicit CRT of the owned quarter, accumulate ----
-    // item m of this thread is entry m of its packed group of every prime
+    // item m of this thread is entry m of its packed group in every prime-CTA
     uint32_t yq[kPrimes][GRP];
 #pragma unroll
     for (int pq = 0; pq < kPrimes; ++pq) {
-      const uint4 w = *reinterpret_cast<const uint4 *>(res + (pq * T + tau) * GRP);
+      const uint4 w = dsmem_ld_v4_u32(HOIST ? res_r[pq] : dsmem_map(res_t, pq));
       yq[pq][0] = w.x;
       yq[pq][1] = w.y;
       yq[pq][2] = w.z;
@@ -351,7 +363,7 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
       const uint32_t u = crt_quotient(ysum);
       acc[c * Q + jl] += s - static_cast<uint64_t>(u) * a.cc.M_mod64;
     }
-    cluster.sync();
+    cluster_sync_shared();
   }
 
   if (a.glwe_out) {
@@ -382,9 +394,8 @@ __global__ void __launch_bounds__(BrShape<LOGN>::T, BrShape<LOGN>::MIN_CTAS) bli
 
 size_t br_smem_bytes(uint32_t logN, uint32_t level, uint32_t n, bool dig16) {
   const size_t N = size_t(1) << logN, Q = N / 4;
-  const size_t xbuf = br_xbuf(static_cast<int>(logN));
-  size_t b = N * sizeof(uint2) + 2 * Q * sizeof(uint64_t) + kPrimes * 2 * Q * sizeof(uint32_t) +
-             xbuf * (N + N / 8) * sizeof(uint32_t) + 2 * level * Q * (dig16 ? 2 : 4) + (n + 1) * sizeof(uint16_t);
+  size_t b = N * sizeof(uint2) + 2 * Q * sizeof(uint64_t) + br_xb_words(static_cast<int>(logN)) * sizeof(uint32_t) +
+             2 * level * Q * (dig16 ? 2 : 4) + (n + 1) * sizeof(uint16_t);
   return (b + 15) & ~size_t(15);
 }
 

@@ -21,6 +21,8 @@
 //     registers across the cluster barrier (its threads are their owners) and
 //     leaves every other owner's slots, one packed group per thread, in its
 //     own exchange buffer, from which the owners read them in phase 3.
+// Every cross-CTA read follows a write to the writer's own shared memory, so
+// the step's barriers order shared memory only (cluster_sync_shared).
 // Per ciphertext and step the cluster runs 3 (l + 1) x 2 transforms instead
 // of 4 (l + 1) x 2; a butterfly is seven instructions instead of five and,
 // measured alone, about 15 % slower.
@@ -217,7 +219,7 @@ __global__ void __launch_bounds__(Br3Shape<LOGN>::T, Br3Shape<LOGN>::MIN_CTAS) b
         if (three) dig4[P * T + tau] = pack16(g[P][0][2], g[P][1][2]);
       }
     }
-    cluster.sync();
+    cluster_sync_shared();
 
     // ---- phase 2: transforms and pointwise products for prime `rank` ----
     uint32_t oh[2][E];
@@ -293,7 +295,7 @@ __global__ void __launch_bounds__(Br3Shape<LOGN>::T, Br3Shape<LOGN>::MIN_CTAS) b
       yo[c][1] = rank == 0 ? oh[c][1] : (rank == 1 ? oh[c][4] : oh[c][7]);
       yo[c][2] = rank == 0 ? oh[c][2] : oh[c][5];
     }
-    cluster.sync();
+    cluster_sync_shared();
 
     // ---- phase 3: explicit CRT of the owned slots, accumulate ----
     {
@@ -324,7 +326,7 @@ __global__ void __launch_bounds__(Br3Shape<LOGN>::T, Br3Shape<LOGN>::MIN_CTAS) b
           acc[(c * 3 + h) * T + tau] += s - static_cast<uint64_t>(u) * a.cc.M_mod64;
         }
     }
-    cluster.sync();
+    cluster_sync_shared();
   }
 
   if (a.glwe_out) {

@@ -17,6 +17,24 @@ __device__ __forceinline__ uint32_t dsmem_map(uint32_t local, uint32_t rank) {
   return r;
 }
 
+// Cluster barrier that orders shared memory only: each thread's earlier
+// writes to its own CTA's shared memory are visible to the reads that the
+// cluster's CTAs make through distributed shared memory after the barrier.
+// The plain cluster barrier (release and acquire at cluster scope) orders
+// global memory as well, which the blind-rotation step loops never need
+// across a barrier (their global accesses read keys and inputs only); a
+// release fence restricted to shared::cta before a relaxed arrive, and an
+// acquire fence restricted to shared::cluster after the wait, give the
+// ordering they do need.  Valid only where every write before the barrier
+// that a remote CTA reads after it went to the writer's own shared memory.
+__device__ __forceinline__ void cluster_sync_shared() {
+  asm volatile(
+      "fence.release.sync_restrict::shared::cta.cluster;\n\t"
+      "barrier.cluster.arrive.relaxed.aligned;\n\t"
+      "barrier.cluster.wait.aligned;\n\t"
+      "fence.acquire.sync_restrict::shared::cluster.cluster;" ::: "memory");
+}
+
 __device__ __forceinline__ uint64_t dsmem_ld_u64(uint32_t a) {
   uint64_t v;
   asm volatile("ld.shared::cluster.u64 %0, [%1];" : "=l"(v) : "r"(a) : "memory");

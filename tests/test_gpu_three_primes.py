@@ -47,9 +47,11 @@ def _br3_smem(N, level, n):
 
 
 def _br4_smem(N, level, n):
-    """Shared memory of one four-prime CTA with 16-bit digits (N >= 2048)."""
+    """Shared memory of one four-prime CTA with 16-bit digits (N >= 2048):
+    twiddles, accumulator quarter, the exchange buffer of 2N words that also
+    holds the outgoing residues, digits, the switched mask."""
     Q = N // 4
-    b = 8 * N + 16 * Q + 32 * Q + 4 * (N + N // 8) + 4 * level * Q + 2 * (n + 1)
+    b = 8 * N + 16 * Q + 8 * N + 4 * level * Q + 2 * (n + 1)
     return (b + 15) & ~15
 
 
@@ -86,7 +88,7 @@ def test_rule_at_the_bound_and_at_the_shared_memory_limit():
         pytest.skip("this torch does not report shared memory per SM")
     fits = lambda b: per_sm // (b + 1024)
     for N, beta, level in ((4096, 15, 2), (8192, 14, 3)):
-        top = 12000 if N == 4096 else 3583                        # the four-prime kernel's own n limit
+        top = 14000 if N == 4096 else 22015                       # beyond: the four-prime kernel's own limit
         rule = [fits(_br3_smem(N, level, n)) >= fits(_br4_smem(N, level, n)) for n in range(1, top + 1)]
         flips = [n for n in range(2, top + 1) if rule[n - 1] != rule[n - 2]]
         for n in sorted({1, top} | {m for f in flips for m in (f - 1, f)}):

@@ -47,6 +47,7 @@ VARIANTS = [
     (2048, 16, 1), (2048, 13, 2), (2048, 11, 3), (2048, 16, 4), (2048, 28, 1), (2048, 24, 2), (2048, 21, 3),
     (4096, 16, 1), (4096, 12, 2), (4096, 11, 3), (4096, 9, 5), (4096, 28, 1), (4096, 24, 2), (4096, 21, 3),
     (8192, 16, 1), (8192, 10, 2), (8192, 15, 2), (8192, 16, 3), (8192, 28, 1),
+    (8192, 12, 4), (8192, 20, 2), (8192, 17, 3),
 ]
 
 
@@ -62,12 +63,14 @@ def test_every_specialisation_bitexact(N, base_log, level):
     assert np.array_equal(got, O.blind_rotate_extract_batch(p, bsk, lwe, lut))
 
 
-@pytest.mark.parametrize("N,base_log,level,n", [(8192, 12, 4, 2), (8192, 20, 2, 2), (8192, 17, 3, 2),
-                                                 (8192, 14, 3, 3584)])
+@pytest.mark.parametrize("N,base_log,level,n", [(8192, 14, 3, 22016), (8192, 12, 4, 17920), (8192, 20, 2, 17920),
+                                                 (8192, 17, 3, 9728)])
 def test_parameter_sets_beyond_shared_memory_are_refused(N, base_log, level, n):
-    """At N = 8192 the CTA (twiddles, accumulator quarter, residues, one
-    exchange buffer: 196 KB) leaves room for the digits of l <= 3 levels of
-    16-bit digits or one level of 32-bit digits, and the a~_i of n <= 3583."""
+    """At N = 8192 the four-prime CTA (twiddles 64 KB, accumulator quarter
+    32 KB, exchange buffer 64 KB) leaves 72 KB of the 227 KB a CTA may have
+    for the digits (8 KB per level of 16-bit digits, 16 KB of 32-bit ones)
+    and the a~_i (2 bytes each): the first n past the limit is refused, the
+    one before it accepted."""
     import paper_2609_16915_gb300 as R
     with pytest.raises(R.RosettaError) as e:
         R.Context(_params(N, base_log, level, n), device=0)

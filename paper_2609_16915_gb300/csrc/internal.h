@@ -81,6 +81,23 @@ struct TraceArgs {
   CrtConsts cc;
 };
 
+// Cluster placement of a blind-rotation launch of `ctas` CTAs: packed onto
+// the SMs with room (load-balancing) once the launch fills every CTA slot of
+// the GPU at least once, spread over the SMs below that.  Measured on GB300:
+// load-balancing is 2-2.5 % faster for full batches and 5.6 % slower for a
+// partial wave (256 CTAs of the standard set).
+template <typename K>
+inline cudaClusterSchedulingPolicy br_cluster_policy(K kern, int threads, size_t smem, size_t ctas) {
+  int dev = 0, sms = 0, per_sm = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, threads, smem) != cudaSuccess) {
+    cudaGetLastError();  // the query's own error; the launch decides the rest
+    return cudaClusterSchedulingPolicySpread;
+  }
+  return ctas >= static_cast<size_t>(sms) * static_cast<size_t>(per_sm) ? cudaClusterSchedulingPolicyLoadBalancing
+                                                                        : cudaClusterSchedulingPolicySpread;
+}
+
 // host-side tables (tables.cu): twiddles and CRT constants of the 28-bit set
 // (primes = kPrimes) or of the 31-bit set (primes = kPrimes31)
 bool build_tables(uint32_t logN, uint32_t primes, uint2 *tw_host /*[primes][N]*/, CrtConsts *cc);

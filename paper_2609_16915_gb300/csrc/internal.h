@@ -17,8 +17,8 @@ constexpr uint32_t kPrimeList[kPrimes] = {268369921u, 268271617u, 268238849u, 26
 // Three NTT primes p = c * 2^14 + 1 in (2^31 - 2^19, 2^31), product
 // M > 2^92.999: the blind rotation's prime set for the parameter sets whose
 // external-product bound stays below 0.45 M (N = 4096 with (k+1) l 2^beta up
-// to 2^17, e.g. l = 2, beta = 15).  No lazy headroom (4p > 2^32): residues are
-// kept in [0, 2p).
+// to 2^17, e.g. l = 2, beta = 15; N = 8192 up to 2^16.8, e.g. l = 3,
+// beta = 14).  No lazy headroom (4p > 2^32): residues are kept in [0, 2p).
 constexpr int kPrimes31 = 3;
 constexpr uint32_t kPrime31List[kPrimes31] = {2147352577u, 2147205121u, 2147074049u};
 
